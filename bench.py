@@ -1,0 +1,493 @@
+"""Benchmark: pattern- and connectivity-pruned 3x3 conv networks on one GB300.
+
+Default workload: the VGG-16 conv trunk at 1x3x224x224 fp32 (13 pattern-pruned
+convs, bias+ReLU, 4 fused 2x2 pools; conv1 keeps all kernels, the rest 30%).
+A step is one frame through the whole trunk with ``pp_net_run`` (CUDA-graph
+replay), inputs resident in HBM, L2 flushed between steps.
+
+Printed JSON line (rank 0):
+  value      surviving-weight GFLOP/s over all ranks (2 FLOP per kept MAC of the
+             4 pattern taps; pruned kernels and taps never counted)
+  ms_per_step  ms per frame
+  e2e        the same metric through pp_net_run_host (pinned host buffers,
+             H2D + run + D2H + sync every step)
+  roofline   the pruned-conv kernel: achieved TFLOP/s over its launches vs the
+             FP32 FMA peak 152 SM x 128 lanes x 2 FLOP x 2.07 GHz
+  cpu_baseline the fp64 CPU oracle on this host's cores on a bounded sample
+  configs    ms/frame, GFLOP/s and roofline fraction of all five workloads
+
+``--impl reference`` times the CPU oracle alone (the reference arm of this
+build: the paper ships no code) and prints the same metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+HBM_PEAK_GBS_FALLBACK = 6800.0
+SM_COUNT = 152
+FP32_LANES_PER_SM = 128
+SM_MAX_MHZ = 2070.0
+FP32_PEAK_TFLOPS = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12  # 80.55
+L2_FLUSH_BYTES = 512 << 20
+
+
+def hbm_peak_gbs():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return HBM_PEAK_GBS_FALLBACK, "fallback"
+
+
+# ----------------------------------------------------------------------------- workloads
+
+
+def workload(name: str):
+    from paper_2004_11250_gb300 import synth
+    if name == "vgg16":
+        return synth.cfg1_vgg16()
+    if name == "single":
+        return synth.cfg0_single()
+    if name == "style":
+        return synth.cfg2_style()
+    if name == "vdsr":
+        return synth.cfg3_vdsr()
+    raise ValueError(name)
+
+
+def op_shapes(spec):
+    """Per op: (N, Ci, Co, H, W, Ho, Wo, surviving FLOPs, compulsory bytes, pruned?)."""
+    from paper_2004_11250_gb300 import synth
+    N, C, H, W = spec.x.shape
+    out = []
+    for op in spec.ops:
+        L = op.layer
+        pruned = isinstance(L, synth.PrunedLayer)
+        taps = 4 * L.nk if pruned else 9 * L.Co * L.Ci
+        Ho, Wo = (H // 2, W // 2) if op.pool else (H, W)
+        flops = 2 * N * H * W * taps
+        nbytes = 4 * N * L.Ci * H * W + 4 * N * L.Co * Ho * Wo + 4 * L.Co
+        nbytes += 21 * L.nk if pruned else 36 * L.Co * L.Ci
+        if op.skip_from >= 0:
+            nbytes += 4 * N * L.Co * H * W
+        out.append(dict(N=N, Ci=L.Ci, Co=L.Co, H=H, W=W, Ho=Ho, Wo=Wo, flops=flops, bytes=nbytes, pruned=pruned))
+        H, W = Ho, Wo
+    return out
+
+
+def roof_time_s(flops, nbytes, hbm):
+    return max(flops / (FP32_PEAK_TFLOPS * 1e12), nbytes / (hbm * 1e9))
+
+
+# ----------------------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    """nvidia-smi sampling (200 ms) during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": float(rows[0][2]) if rows[0][2].replace(".", "").isdigit() else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle baseline
+
+
+def cpu_oracle_sample(spec, target_s: float, seed: int = 0):
+    """Time the fp64 oracle on a bounded sample of the workload: every op, restricted to its first
+    ceil(f * Co) filters, on a seeded input of the op's input shape.  f is calibrated on the first
+    pruned op so that the whole sample takes about target_s seconds.  Returns (GFLOP/s, f, seconds)."""
+    from oracle import oracle as orc
+    from paper_2004_11250_gb300 import synth
+    rng = np.random.default_rng(seed)
+    shapes = op_shapes(spec)
+    total_flops = sum(s["flops"] for s in shapes)
+    inputs = [rng.uniform(-1, 1, (s["N"], s["Ci"], s["H"], s["W"])).astype(np.float32) for s in shapes]
+    pats = [orc.pattern_ids(op.layer.w, op.layer.mask, op.layer.taps) if isinstance(op.layer, synth.PrunedLayer)
+            else None for op in spec.ops]
+
+    def run(k, f):
+        L = spec.ops[k].layer
+        co = max(1, int(math.ceil(f * L.Co)))
+        t0 = time.perf_counter()
+        if pats[k] is not None:
+            orc.conv_pruned(inputs[k], L.w[:co], pats[k][:co], L.taps, None if L.bias is None else L.bias[:co])
+        else:
+            orc.conv_dense(inputs[k], L.w[:co], None if L.bias is None else L.bias[:co])
+        dt = time.perf_counter() - t0
+        s = shapes[k]
+        return dt, s["flops"] * co / s["Co"]
+
+    k0 = max(range(len(shapes)), key=lambda k: shapes[k]["flops"])
+    f0 = min(1.0, 2.0 / max(1, shapes[k0]["Co"]))
+    dt, fl = run(k0, f0)
+    rate = fl / max(dt, 1e-9)
+    f = min(1.0, target_s * rate / total_flops)
+    t_all, fl_all = 0.0, 0.0
+    for k in range(len(shapes)):
+        dt, fl = run(k, f)
+        t_all += dt
+        fl_all += fl
+    return fl_all / t_all / 1e9, f, t_all
+
+
+# ----------------------------------------------------------------------------- GPU timing
+
+
+def time_net(dn, x, y, steps, warmup, flush, stream):
+    import torch
+    for _ in range(warmup):
+        flush.zero_()
+        dn.run(x, y, stream)
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for e0, e1 in evs:
+        flush.zero_()
+        e0.record(stream)
+        dn.run(x, y, stream)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return [e0.elapsed_time(e1) for e0, e1 in evs]
+
+
+def time_ops(dn, acts, steps, flush, stream):
+    """Average duration (ms) of every op's kernel launch, L2 flushed before each launch."""
+    import torch
+    from paper_2004_11250_gb300 import runner
+    spec = dn.spec
+    res = []
+    for k, (op, L) in enumerate(zip(spec.ops, dn.layers)):
+        xin, out = acts[k], acts[k + 1]
+        skip = acts[op.skip_from] if op.skip_from >= 0 else None
+        N, _, H, W = xin.shape
+        flags = runner.op_flags(op)
+        L.forward(xin, out, skip, N, H, W, flags, stream)
+        ts = []
+        for _ in range(steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            L.forward(xin, out, skip, N, H, W, flags, stream)
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        res.append(sum(ts) / len(ts))
+    return res
+
+
+def traffic_from_profile(kernel_hash: str):
+    """Per-launch DRAM bytes of the pruned-conv kernel from the committed ncu summary, if that summary
+    was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "ppconv_vgg16_dram_traffic.txt")
+    try:
+        kv = {}
+        for line in open(path):
+            if ":" in line:
+                k, v = line.split(":", 1)
+                kv[k.strip()] = v.strip()
+        if kv.get("kernel_source_sha256") != kernel_hash:
+            return None
+        return float(kv["dram_bytes_per_launch_avg"])
+    except Exception:
+        return None
+
+
+def kernel_source_hash():
+    import hashlib
+    with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", "conv.cu"), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def bench_config(name, steps, warmup, flush, stream, hbm):
+    """ms/frame, GFLOP/s and per-op roofline fractions of one workload (used for the all-configs table)."""
+    import torch
+    from paper_2004_11250_gb300 import runner
+    spec = workload(name)
+    dn = runner.DeviceNet(spec, use_graph=True)
+    try:
+        x = torch.from_numpy(spec.x).cuda()
+        y = torch.empty(dn.out_shape, device="cuda")
+        ts = time_net(dn, x, y, steps, warmup, flush, stream)
+        shapes = op_shapes(spec)
+        acts = dn.run_layerwise(x)
+        op_ms = time_ops(dn, acts, max(3, steps // 2), flush, stream)
+        flops = sum(s["flops"] for s in shapes)
+        ms = statistics.median(ts)
+        fr = [roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3) for s, t in zip(shapes, op_ms)]
+        pr = [f for s, f in zip(shapes, fr) if s["pruned"]]
+        del acts
+        return {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1),
+                "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
+                "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None}
+    finally:
+        dn.close()
+
+
+def bench_sweep(steps, flush, stream, hbm):
+    """Sweep workload: per point (C, P, keep) one layer at 8x56x56; returns summary + per-point fracs."""
+    import torch
+    from paper_2004_11250_gb300 import runner, synth
+    fracs, total_ms = {}, 0.0
+    for (C, P, keep) in synth.cfg4_points():
+        spec = synth.cfg4_point(C, P, keep)
+        L = runner.DeviceLayer(spec.ops[0].layer)
+        try:
+            x = torch.from_numpy(spec.x).cuda()
+            y = torch.empty((8, C, 56, 56), device="cuda")
+            L.forward(x, y, None, 8, 56, 56, 0, stream)
+            ts = []
+            for _ in range(steps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                L.forward(x, y, None, 8, 56, 56, 0, stream)
+                e1.record(stream)
+                e1.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            t = statistics.median(ts)
+            s = op_shapes(spec)[0]
+            fracs[f"C{C}_P{P}_k{keep}"] = round(roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3), 3)
+            total_ms += t
+        finally:
+            L.close()
+    v = list(fracs.values())
+    return {"points": len(v), "ms_total": round(total_ms, 3), "roofline_frac_min": min(v),
+            "roofline_frac_median": statistics.median(v), "per_point": fracs}
+
+
+# ----------------------------------------------------------------------------- main
+
+
+def dist_setup(args):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        backend = "nccl" if args.impl != "reference" else "gloo"
+        dist.init_process_group(backend)
+    return ws, rank, local
+
+
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return
+    from oracle import oracle as orc
+    spec = workload(args.workload)
+    per_step = max(1.0, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        cpu_oracle_sample(spec, per_step)
+    vals, fs = [], []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        v, f, _ = cpu_oracle_sample(spec, per_step)
+        vals.append(v)
+        fs.append(f)
+    wall = time.perf_counter() - t0
+    value = statistics.median(vals)
+    flops = sum(s["flops"] for s in op_shapes(spec))
+    line = {
+        "impl": "reference", "metric": metric_name(args.workload), "value": round(value, 3), "unit": "GFLOP/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(flops / (value * 1e9) * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_dict(args.workload),
+        "cpu_baseline": {"value": round(value, 3), "unit": "GFLOP/s", "cores": orc.num_threads(), "kind": "oracle",
+                         "sample": f"every op of the workload on its first {statistics.median(fs):.4f} of filters, "
+                                   f"seeded inputs; {wall:.1f} s for {args.steps} steps"},
+        "e2e": {"value": round(value, 3), "unit": "GFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def metric_name(w):
+    names = {"vgg16": "VGG-16 pattern-pruned conv trunk 1x3x224x224",
+             "single": "single pattern-pruned layer 1x16x32x32",
+             "style": "style-transfer residual trunk 1x128x128x128",
+             "vdsr": "VDSR-shaped SR stack 1x1x720x1280"}
+    return f"effective GFLOP/s (surviving MACs), {names[w]}, fp32"
+
+
+def config_dict(w):
+    from paper_2004_11250_gb300 import synth
+    spec = workload(w)
+    return {"workload": metric_name(w).split(", ")[1], "batch": int(spec.x.shape[0]),
+            "input": list(spec.x.shape), "convs": len(spec.ops),
+            "surviving_gflop_per_frame": round(spec.surviving_flops() / 1e9, 4),
+            "patterns": "8 fixed centre+3-neighbour patterns", "l2": "flushed between steps (512 MiB write)"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="vgg16", choices=["vgg16", "single", "style", "vdsr"])
+    ap.add_argument("--no-configs", action="store_true", help="skip the all-configs table")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    ws, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2004_11250_gb300 import build
+    build.build()
+    from paper_2004_11250_gb300 import runner
+    hbm, hbm_src = hbm_peak_gbs()
+    stream = torch.cuda.Stream()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    spec = workload(args.workload)
+    shapes = op_shapes(spec)
+    flops_frame = sum(s["flops"] for s in shapes)
+    dn = runner.DeviceNet(spec, use_graph=True)
+    x = torch.from_numpy(spec.x).cuda()
+    y = torch.empty(dn.out_shape, device="cuda")
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    with torch.cuda.stream(stream):
+        if ws > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        clocks.start()
+        ts = time_net(dn, x, y, args.steps, args.warmup, flush, stream)
+        torch.cuda.synchronize()
+        clk = clocks.stop()
+    t_total_ms = sum(ts)
+    if ws > 1:
+        t = torch.tensor([t_total_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        t_total_ms = float(t.item())
+        torch.distributed.barrier()
+    ms_per_step = t_total_ms / args.steps
+    value = ws * flops_frame * args.steps / (t_total_ms * 1e-3) / 1e9
+
+    # per-op kernel durations (same stream, L2 flushed before each launch) -> roofline of the pruned conv
+    acts = dn.run_layerwise(x, stream)
+    torch.cuda.synchronize()
+    op_ms = time_ops(dn, acts, max(5, args.steps // 2), flush, stream)
+    del acts
+    pruned = [k for k, s in enumerate(shapes) if s["pruned"]]
+    kf = sum(shapes[k]["flops"] for k in pruned)
+    kt = sum(op_ms[k] for k in pruned) * 1e-3
+    achieved = kf / kt / 1e12
+    traffic = traffic_from_profile(kernel_source_hash())
+    layer_fracs = [round(roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3), 3) for s, t in zip(shapes, op_ms)]
+
+    # end to end through the public API with host buffers
+    xh = torch.from_numpy(spec.x).pin_memory()
+    yh = torch.empty(dn.out_shape, dtype=torch.float32).pin_memory()
+    for _ in range(args.warmup):
+        dn.run_host(xh, yh, stream)
+    e2e_t = []
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dn.run_host(xh, yh, stream)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_value = ws * flops_frame / statistics.median(e2e_t) / 1e9
+
+    configs = None
+    if not args.no_configs and rank == 0:
+        configs = {}
+        for name in ("single", "vgg16", "style", "vdsr"):
+            configs[name] = bench_config(name, 10, 3, flush, stream, hbm)
+        configs["sweep"] = bench_sweep(5, flush, stream, hbm)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu:
+        from oracle import oracle as orc
+        v, f, secs = cpu_oracle_sample(spec, args.cpu_seconds)
+        cpu = {"value": round(v, 3), "unit": "GFLOP/s", "cores": orc.num_threads(), "kind": "oracle",
+               "sample": f"every op on its first {f:.4f} of filters (seeded inputs), {secs:.1f} s"}
+
+    if rank == 0:
+        line = {
+            "metric": metric_name(args.workload), "value": round(value, 2), "unit": "GFLOP/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded; shapes and distributions of the workload, no dataset or trained weights)",
+            "config": config_dict(args.workload),
+            "e2e": {"value": round(e2e_value, 2), "unit": "GFLOP/s", "h2d_bytes_per_step": int(xh.numel() * 4),
+                    "d2h_bytes_per_step": int(yh.numel() * 4), "ms_per_step": round(statistics.median(e2e_t) * 1e3, 4)},
+            "gpu_launches": len(spec.ops) * args.steps,
+            "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
+                         "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
+                         "kernel": "ppconv_kernel (pattern-pruned conv, all pruned ops of a step)",
+                         "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
+                         "hbm_peak_gbs": hbm, "hbm_peak_source": hbm_src},
+            "layer_roofline_frac": layer_fracs,
+            "clocks": clk,
+            "cpu_baseline": cpu,
+            "configs": configs,
+        }
+        print(json.dumps(line), flush=True)
+    dn.close()
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,214 @@
+/*
+ * ppconv.h -- C ABI of a GB300 (sm_103a) library for forward inference of
+ * pattern- and connectivity-pruned 3x3 convolution layers.
+ *
+ * Method: Niu et al., "Towards Real-Time DNN Inference on Mobile Platforms
+ * with Model Pruning and Compiler Optimization" (IJCAI-20 demo).
+ *   Section 2  connectivity pruning removes whole (output, input) kernels;
+ *              pattern pruning keeps certain locations of each kernel: here a
+ *              kept kernel keeps 4 of its 9 taps, forming one pattern of a small
+ *              caller-given pattern set.
+ *   Section 3  "Sparse model storage": zeros and structurally redundant
+ *              indices are not stored; "Matrix reorder": filters are reordered
+ *              so that similar ones sit together, and the kept kernels of each
+ *              filter are compacted; "DSL related optimization": convolution is
+ *              fused with its activation to cut data movement.
+ *
+ * Scope: 3x3 kernels, stride 1, zero padding 1, fp32, NCHW activations.
+ * Anything else is rejected with PP_ERR_UNSUPPORTED.
+ *
+ * Conventions
+ *   - Tap index t = 3*ky + kx (ky, kx in 0..2); weights are [Co][Ci][9].
+ *   - Every function returns a pp_status (0 = PP_OK) unless noted.  Arguments
+ *     are validated on the host before any device work; a call that fails
+ *     validation has no effect.
+ *   - Handles (pp_packed, pp_layer, pp_dense, pp_net) are opaque, created and
+ *     owned by the library, and released with their destroy function
+ *     (destroy(NULL) is a no-op).
+ *   - Device calls take a CUDA stream as `void*` (a cudaStream_t; NULL = the
+ *     legacy default stream), enqueue their work on it and never synchronise
+ *     unless stated.  Launch errors are returned by the call; faults that
+ *     happen later surface at the caller's next synchronisation.
+ *   - Activation, skip and output pointers are caller-owned device memory,
+ *     dense NCHW fp32, 16-byte aligned.  An output must not overlap an input.
+ *   - A handle may be used from one host thread at a time.
+ */
+#ifndef PPCONV_H
+#define PPCONV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum pp_status_code {
+  PP_OK = 0,
+  PP_ERR_INVALID_ARG = 1,        /* null pointer, non-positive size, bad flag  */
+  PP_ERR_BAD_PATTERN_SET = 2,    /* a pattern is not 4 distinct ascending taps in 0..8, or repeats */
+  PP_ERR_TAP_NOT_IN_PATTERN = 3, /* a kept kernel has a nonzero tap outside every pattern */
+  PP_ERR_PRUNED_NONZERO = 4,     /* a connectivity-pruned kernel has a nonzero weight */
+  PP_ERR_PATTERN_ID_MISMATCH = 5,/* a caller-given pattern id does not cover the kernel's taps */
+  PP_ERR_UNSUPPORTED = 6,        /* shape or option outside the library's scope */
+  PP_ERR_CUDA = 7,               /* a CUDA runtime call failed */
+  PP_ERR_OOM = 8                 /* host or device allocation failed */
+};
+typedef int pp_status;
+
+/* Epilogue flags of a convolution, applied in this order after the bias:
+ * add the skip tensor, ReLU, 2x2 max pool (stride 2, floor). */
+#define PP_ADD_SKIP 1
+#define PP_RELU 2
+#define PP_POOL2 4
+
+/* Static string naming a status code ("PP_OK", ...); never NULL. */
+const char* pp_status_string(pp_status status);
+/* Library version: major * 10000 + minor * 100 + patch. */
+int pp_version(void);
+
+/* ------------------------------------------------------------------------
+ * Host packer: compact pattern-grouped storage with filter reorder (Section 3).
+ * ------------------------------------------------------------------------ */
+typedef struct pp_packed pp_packed;
+
+/*
+ * Validate a pruned layer and build its compact form.  Host only, synchronous.
+ *   w            [Co][Ci][9] fp32 host weights; zero outside the kept taps
+ *   mask         [Co][Ci] host bytes, nonzero = kernel kept (connectivity)
+ *   pattern_taps [P][4] host bytes, each row 4 distinct ascending taps in 0..8
+ *   P            number of patterns, 1..126, rows pairwise distinct
+ *   pattern_ids  [Co][Ci] optional (NULL = infer); for each kept kernel, the
+ *                pattern it uses.  Inferred id = lowest pattern containing the
+ *                kernel's nonzero taps.
+ *   out          receives a new handle on success, untouched on failure
+ * Stored form (read with pp_packed_arrays):
+ *   perm[Co]     perm[j] = original index of the j-th filter; filters are
+ *                sorted by (kept count descending, dominant pattern ascending,
+ *                index ascending), the dominant pattern being the most frequent
+ *                pattern id among the filter's kept kernels (lowest on ties)
+ *   kptr[Co+1]   kept kernels of filter perm[j] are entries kptr[j]..kptr[j+1]-1
+ *   kidx[nk]     input channel of each entry
+ *   kpat[nk]     pattern id of each entry
+ *   kw[nk][4]    weights on the pattern's taps in ascending tap order
+ *   Entries of a filter are ordered by (pattern id, input channel).
+ * Errors: PP_ERR_INVALID_ARG, PP_ERR_BAD_PATTERN_SET, PP_ERR_PRUNED_NONZERO,
+ *   PP_ERR_TAP_NOT_IN_PATTERN, PP_ERR_PATTERN_ID_MISMATCH, PP_ERR_OOM.
+ */
+pp_status pp_pack_layer(const float* w, const uint8_t* mask, const uint8_t* pattern_taps, int P, int Co, int Ci,
+                        const uint8_t* pattern_ids, pp_packed** out);
+
+/* Sizes of a packed layer; any output pointer may be NULL. */
+pp_status pp_packed_info(const pp_packed* pk, int64_t* nk, int* Co, int* Ci, int* P);
+
+/* Borrowed read-only views of the stored arrays (valid until destroy); any
+ * output pointer may be NULL.  taps is the [P][4] pattern set. */
+pp_status pp_packed_arrays(const pp_packed* pk, const int32_t** perm, const int32_t** kptr, const int32_t** kidx,
+                           const uint8_t** kpat, const float** kw, const uint8_t** taps);
+
+/* Rebuild the dense weights [Co][Ci][9] and mask [Co][Ci] (host buffers; either
+ * may be NULL).  Kept taps come back bit for bit, every other tap as +0.0. */
+pp_status pp_unpack_layer(const pp_packed* pk, float* w_out, uint8_t* mask_out);
+
+void pp_packed_destroy(pp_packed* pk);
+
+/* ------------------------------------------------------------------------
+ * Device layer: the pruned convolution on the GPU (Sections 2-3).
+ * ------------------------------------------------------------------------ */
+typedef struct pp_layer pp_layer;
+
+/*
+ * Upload a packed layer to the current CUDA device.  The library allocates
+ * and owns the device copy (a few bytes per kept kernel) and derives its
+ * kernel-side layout from pk; pk may be destroyed afterwards.
+ *   bias   [Co] host fp32 or NULL (no bias)
+ *   stream copies are enqueued on it; the call waits for them before returning
+ * Errors: PP_ERR_INVALID_ARG, PP_ERR_UNSUPPORTED, PP_ERR_CUDA, PP_ERR_OOM.
+ */
+pp_status pp_layer_create(const pp_packed* pk, const float* bias, void* stream, pp_layer** out);
+
+/* Co, Ci and the number of device bytes held by the layer (any may be NULL). */
+pp_status pp_layer_info(const pp_layer* layer, int* Co, int* Ci, int64_t* device_bytes);
+
+/*
+ * y = epilogue(conv(x) + bias): the pruned 3x3 convolution of every image of
+ * the batch, fused with the epilogue given by flags (PP_ADD_SKIP, PP_RELU,
+ * PP_POOL2, in that order).  Asynchronous on stream.
+ *   x     [N][Ci][H][W] device input
+ *   y     [N][Co][H][W], or [N][Co][H/2][W/2] with PP_POOL2 (H, W even)
+ *   skip  [N][Co][H][W] device tensor added before the ReLU (PP_ADD_SKIP), else NULL
+ * Errors: PP_ERR_INVALID_ARG (null pointer, N/H/W < 1, flags), PP_ERR_UNSUPPORTED
+ *   (PP_POOL2 with odd H or W, or a pattern the kernels do not cover),
+ *   PP_ERR_CUDA (launch failure).
+ */
+pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H, int W,
+                          int flags, void* stream);
+
+void pp_layer_destroy(pp_layer* layer);
+
+/* ------------------------------------------------------------------------
+ * Dense (unpruned) 3x3 layer, for the end layers of a pruned network.
+ * ------------------------------------------------------------------------ */
+typedef struct pp_dense pp_dense;
+
+/* w [Co][Ci][9] and bias [Co] (or NULL) are host fp32; copied to the device. */
+pp_status pp_dense_create(const float* w, const float* bias, int Co, int Ci, void* stream, pp_dense** out);
+
+/* Same contract as pp_conv_forward, over all 9 taps of every kernel. */
+pp_status pp_dense_forward(const pp_dense* layer, const float* x, float* y, const float* skip, int N, int H, int W,
+                           int flags, void* stream);
+
+/* Co and Ci of a dense layer (either may be NULL). */
+pp_status pp_dense_info(const pp_dense* layer, int* Co, int* Ci);
+
+void pp_dense_destroy(pp_dense* layer);
+
+/* ------------------------------------------------------------------------
+ * Network executor: a chain of convolutions on one stream (Section 3's
+ * layer-wise representation, run as a fixed schedule).
+ * ------------------------------------------------------------------------ */
+typedef struct pp_net pp_net;
+
+/* An empty network for inputs [N][C][H][W]. */
+pp_status pp_net_create(int N, int C, int H, int W, pp_net** out);
+
+/*
+ * Append one op.  Activation 0 is the network input; op k (0-based) writes
+ * activation k + 1.  skip_from = index of an earlier activation added before
+ * the ReLU (requires PP_ADD_SKIP in flags and the same shape), or -1.
+ * The layer handle is borrowed: it must outlive the network.
+ */
+pp_status pp_net_add_conv(pp_net* net, const pp_layer* layer, int flags, int skip_from);
+pp_status pp_net_add_dense(pp_net* net, const pp_dense* layer, int flags, int skip_from);
+
+/* Plan activation buffers and allocate them on the current device (library
+ * owned).  Must be called once, after the last add and before the first run. */
+pp_status pp_net_finalize(pp_net* net);
+
+/* Shape of the network output (any pointer may be NULL). */
+pp_status pp_net_output_shape(const pp_net* net, int* N, int* C, int* H, int* W);
+
+/* With enable != 0, pp_net_run captures its launches into a CUDA graph on the
+ * first call for a given (x, y, stream) and replays that graph afterwards (one
+ * host launch per run).  Needs a non-NULL stream; with the legacy default
+ * stream the ops are launched one by one.  Default: off. */
+pp_status pp_net_use_graph(pp_net* net, int enable);
+
+/* Device-resident run: x and y are device buffers of the input and output
+ * shapes.  Launches every op on stream; asynchronous. */
+pp_status pp_net_run(pp_net* net, const float* x, float* y, void* stream);
+
+/*
+ * End-to-end run on host buffers: copies x_host to the device, runs the
+ * network and copies the output to y_host, all on stream, and synchronises
+ * the stream before returning.  Pinned host memory gives overlap-free DMA at
+ * full speed; pageable memory works too.
+ */
+pp_status pp_net_run_host(pp_net* net, const float* x_host, float* y_host, void* stream);
+
+void pp_net_destroy(pp_net* net);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PPCONV_H */

@@ -1,0 +1,567 @@
+// Pattern- and connectivity-pruned 3x3 convolution on sm_103a (FP32 SIMT).
+//
+// Method: Niu et al., IJCAI-20 demo.  Section 2: a kept kernel keeps 4 of its 9
+// taps (one pattern of a small set); connectivity pruning drops whole kernels.
+// Section 3: compact storage (pattern id + 4 weights per kept kernel), filter
+// reorder so similar filters sit together, and convolution fused with its
+// activation.
+//
+// Kernel design (GB300-first, not the paper's mobile code generator):
+//   * A warp owns kSlots consecutive reordered filters ("slots") and a 16x16
+//     output tile; a lane owns one row segment of 8 pixels, so its
+//     accumulators are acc[16][8] registers, indexed only by compile-time
+//     constants.
+//   * Input channels are staged 16 at a time into shared memory (tile + 1-pixel
+//     halo, zero padding) with cp.async, double buffered.
+//   * Per input channel a lane loads its 3x10 input window once into
+//     registers and reuses it for every kept kernel of that channel in its
+//     filter group: this reuse across filters is what keeps the FMA pipe fed
+//     instead of the shared-memory port.
+//   * The kept kernels of a warp's filter group form one entry stream, sorted
+//     by input channel (the reorder and compaction of Section 3 decide which
+//     filters share a stream and keep adjacent streams equally long).  An
+//     entry is (channel, slot, pattern) + 4 weights; the (slot, pattern) pair
+//     selects a fully unrolled 4-tap x 8-pixel FMA block through one
+//     warp-uniform switch.  For the ring set of 8 centre-based patterns the
+//     taps are compile-time constants; any other pattern set goes through a
+//     per-tap switch (slower, same results).
+//   * Epilogue: bias, optional residual add, ReLU, optional 2x2 max pool (the
+//     partner row comes from the neighbouring lane by shuffle), store to the
+//     filter's original channel.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "internal.h"
+
+namespace {
+
+constexpr int F = ppc::kSlots;   // filter slots per warp
+constexpr int PX = 8;            // pixels per lane (one row segment)
+constexpr int TH = 16;           // output tile rows (lanes 0..15 of a half)
+constexpr int TW = 16;           // output tile cols (2 lane columns x 8)
+constexpr int NWF = 4;           // warps (filter groups) per CTA
+constexpr int CC = ppc::kChunk;  // input channels per stage
+constexpr int SROWS = TH + 2;
+constexpr int SCOLS = TW + 2;
+constexpr int SSTRIDE = 20;      // row stride (floats): 16B aligned, conflict-free LDS.128 per 8-lane phase
+constexpr int SCH = SROWS * SSTRIDE;
+constexpr int STAGE = CC * SCH;
+constexpr int NTHREADS = 32 * NWF;
+
+enum Mode { MODE_RING8 = 0, MODE_GENERIC = 1 };
+
+// The ring set: centre (tap 4) plus 3 consecutive neighbours in the ring order
+// 0,1,2,5,8,7,6,3 around the centre.
+__host__ __device__ constexpr int ring_tap(int r, int s) {
+  // taps of ring pattern r in ascending order
+  return r == 0 ? (s == 0 ? 0 : s == 1 ? 1 : s == 2 ? 2 : 4)
+       : r == 1 ? (s == 0 ? 1 : s == 1 ? 2 : s == 2 ? 4 : 5)
+       : r == 2 ? (s == 0 ? 2 : s == 1 ? 4 : s == 2 ? 5 : 8)
+       : r == 3 ? (s == 0 ? 4 : s == 1 ? 5 : s == 2 ? 7 : 8)
+       : r == 4 ? (s == 0 ? 4 : s == 1 ? 6 : s == 2 ? 7 : 8)
+       : r == 5 ? (s == 0 ? 3 : s == 1 ? 4 : s == 2 ? 6 : 7)
+       : r == 6 ? (s == 0 ? 0 : s == 1 ? 3 : s == 2 ? 4 : 6)
+       :          (s == 0 ? 0 : s == 1 ? 1 : s == 2 ? 3 : 4);
+}
+
+struct ConvParams {
+  const float* x;        // [N][Ci][H][W]
+  float* y;              // [N][Co][H'][W']
+  const float* skip;     // [N][Co][H][W] or null
+  const int* cofs;       // [G][nch + 1] entry offsets per (group, chunk)
+  const uint32_t* code;  // [nE]
+  const float4* wts;     // [nE]
+  const int* perm;       // [Co]
+  const float* bias;     // [Co] in reordered order, or null
+  int N, Ci, Co, H, W;
+  int nch, G;
+  int tiles_x;
+  int flags;
+};
+
+// Entry code layout: bits 0..15 pattern payload (MODE_RING8: ring index;
+// MODE_GENERIC: 4 taps x 4 bits), 16..19 slot, 20..27 channel within the stage,
+// 28..29 number of taps - 1 (MODE_GENERIC).
+__device__ __forceinline__ int code_slot(uint32_t c) { return (c >> 16) & 15; }
+__device__ __forceinline__ int code_ch(uint32_t c) { return (c >> 20) & 255; }
+
+template <int T>
+__device__ __forceinline__ void tap_fma(float (&a)[PX], const float (&win)[3][PX + 2], float w) {
+  constexpr int dy = T / 3, dx = T % 3;
+#pragma unroll
+  for (int k = 0; k < PX; ++k) a[k] = fmaf(w, win[dy][k + dx], a[k]);
+}
+
+template <int R>
+__device__ __forceinline__ void ring_fma(float (&a)[PX], const float (&win)[3][PX + 2], const float4& w) {
+  tap_fma<ring_tap(R, 0)>(a, win, w.x);
+  tap_fma<ring_tap(R, 1)>(a, win, w.y);
+  tap_fma<ring_tap(R, 2)>(a, win, w.z);
+  tap_fma<ring_tap(R, 3)>(a, win, w.w);
+}
+
+__device__ __forceinline__ void cp_async4(float* sdst, const float* gsrc, bool valid) {
+  unsigned saddr = (unsigned)__cvta_generic_to_shared(sdst);
+  int n = valid ? 4 : 0;
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(saddr), "l"(gsrc), "r"(n));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+
+// Stage channels [i0, i0 + nvalid) of image n, rows r0-1..r0+TH, cols c0-1..c0+TW.
+__device__ __forceinline__ void stage_chunk(float* s, const ConvParams& p, int n, int i0, int nvalid, int r0,
+                                            int c0) {
+  const int total = nvalid * SROWS * SCOLS;
+  const float* xb = p.x + ((size_t)n * p.Ci + i0) * p.H * p.W;
+  for (int e = threadIdx.x; e < total; e += NTHREADS) {
+    const int ch = e / (SROWS * SCOLS);
+    const int rem = e - ch * (SROWS * SCOLS);
+    const int sr = rem / SCOLS;
+    const int sc = rem - sr * SCOLS;
+    const int r = r0 - 1 + sr, c = c0 - 1 + sc;
+    const bool ok = (unsigned)r < (unsigned)p.H && (unsigned)c < (unsigned)p.W;
+    const float* src = ok ? xb + ((size_t)ch * p.H + r) * p.W + c : p.x;
+    cp_async4(s + ch * SCH + sr * SSTRIDE + sc, src, ok);
+  }
+}
+
+template <int MODE>
+__device__ __forceinline__ void dispatch(float (&acc)[F][PX], const float (&win)[3][PX + 2], uint32_t code,
+                                         float4 w) {
+  if constexpr (MODE == MODE_RING8) {
+    const int cs = code_slot(code) * 8 + (code & 7);
+    switch (cs) {
+#define PP_RING_CASE(J, R) \
+  case (J)*8 + (R): ring_fma<R>(acc[J], win, w); break;
+#define PP_RING_SLOT(J) \
+  PP_RING_CASE(J, 0) PP_RING_CASE(J, 1) PP_RING_CASE(J, 2) PP_RING_CASE(J, 3) \
+  PP_RING_CASE(J, 4) PP_RING_CASE(J, 5) PP_RING_CASE(J, 6) PP_RING_CASE(J, 7)
+      PP_RING_SLOT(0) PP_RING_SLOT(1) PP_RING_SLOT(2) PP_RING_SLOT(3)
+      PP_RING_SLOT(4) PP_RING_SLOT(5) PP_RING_SLOT(6) PP_RING_SLOT(7)
+      PP_RING_SLOT(8) PP_RING_SLOT(9) PP_RING_SLOT(10) PP_RING_SLOT(11)
+      PP_RING_SLOT(12) PP_RING_SLOT(13) PP_RING_SLOT(14) PP_RING_SLOT(15)
+#undef PP_RING_SLOT
+#undef PP_RING_CASE
+      default: break;
+    }
+  } else {
+    const int slot9 = code_slot(code) * 9;
+    const int nt = ((code >> 28) & 3) + 1;
+    uint32_t taps = code & 0xffff;
+    float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll 1
+    for (int s = 0; s < nt; ++s) {
+      const float ws = s == 0 ? wv[0] : s == 1 ? wv[1] : s == 2 ? wv[2] : wv[3];
+      switch (slot9 + (int)(taps & 15)) {
+#define PP_TAP_CASE(J, T) \
+  case (J)*9 + (T): tap_fma<T>(acc[J], win, ws); break;
+#define PP_TAP_SLOT(J) \
+  PP_TAP_CASE(J, 0) PP_TAP_CASE(J, 1) PP_TAP_CASE(J, 2) PP_TAP_CASE(J, 3) PP_TAP_CASE(J, 4) \
+  PP_TAP_CASE(J, 5) PP_TAP_CASE(J, 6) PP_TAP_CASE(J, 7) PP_TAP_CASE(J, 8)
+        PP_TAP_SLOT(0) PP_TAP_SLOT(1) PP_TAP_SLOT(2) PP_TAP_SLOT(3)
+        PP_TAP_SLOT(4) PP_TAP_SLOT(5) PP_TAP_SLOT(6) PP_TAP_SLOT(7)
+        PP_TAP_SLOT(8) PP_TAP_SLOT(9) PP_TAP_SLOT(10) PP_TAP_SLOT(11)
+        PP_TAP_SLOT(12) PP_TAP_SLOT(13) PP_TAP_SLOT(14) PP_TAP_SLOT(15)
+#undef PP_TAP_SLOT
+#undef PP_TAP_CASE
+        default: break;
+      }
+      taps >>= 4;
+    }
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(NTHREADS, 2) ppconv_kernel(const ConvParams p) {
+  __shared__ __align__(16) float smem[2 * STAGE];
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int ly = lane & 15;  // row in tile
+  const int lx = lane >> 4;  // column segment (8 pixels)
+  const int tile = blockIdx.x;
+  const int ty = tile / p.tiles_x, tx = tile - ty * p.tiles_x;
+  const int r0 = ty * TH, c0 = tx * TW;
+  const int n = blockIdx.z;
+  const int q = blockIdx.y * NWF + warp;  // filter group of this warp
+  const bool active = q < p.G;
+
+  float acc[F][PX];
+#pragma unroll
+  for (int j = 0; j < F; ++j)
+#pragma unroll
+    for (int k = 0; k < PX; ++k) acc[j][k] = 0.f;
+
+  const int* cofs = p.cofs + (size_t)(active ? q : 0) * (p.nch + 1);
+
+  stage_chunk(smem, p, n, 0, min(CC, p.Ci), r0, c0);
+  cp_async_commit();
+  for (int c = 0; c < p.nch; ++c) {
+    if (c + 1 < p.nch) {
+      stage_chunk(smem + ((c + 1) & 1) * STAGE, p, n, (c + 1) * CC, min(CC, p.Ci - (c + 1) * CC), r0, c0);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    if (active) {
+      const float* sb = smem + (c & 1) * STAGE + ly * SSTRIDE + lx * PX;
+      const int e0 = __ldg(cofs + c), e1 = __ldg(cofs + c + 1);
+      int cur = -1;
+      float win[3][PX + 2];
+#pragma unroll
+      for (int a = 0; a < 3; ++a)
+#pragma unroll
+        for (int b = 0; b < PX + 2; ++b) win[a][b] = 0.f;
+      for (int e = e0; e < e1; ++e) {
+        const uint32_t code = __ldg(p.code + e);
+        const float4 w = __ldg(p.wts + e);
+        const int ch = code_ch(code);
+        if (ch != cur) {
+          cur = ch;
+          const float* s = sb + ch * SCH;
+#pragma unroll
+          for (int a = 0; a < 3; ++a) {
+            const float4 u = *reinterpret_cast<const float4*>(s + a * SSTRIDE);
+            const float4 v = *reinterpret_cast<const float4*>(s + a * SSTRIDE + 4);
+            const float2 z = *reinterpret_cast<const float2*>(s + a * SSTRIDE + 8);
+            win[a][0] = u.x; win[a][1] = u.y; win[a][2] = u.z; win[a][3] = u.w;
+            win[a][4] = v.x; win[a][5] = v.y; win[a][6] = v.z; win[a][7] = v.w;
+            win[a][8] = z.x; win[a][9] = z.y;
+          }
+        }
+        dispatch<MODE>(acc, win, code, w);
+      }
+    }
+    __syncthreads();
+  }
+  if (!active) return;
+
+  // Epilogue: bias, +skip, ReLU, 2x2 max pool, store at the original channel.
+  const int r = r0 + ly;
+  const int cb = c0 + lx * PX;
+  const bool pool = p.flags & PP_POOL2;
+  const int Ho = pool ? p.H / 2 : p.H, Wo = pool ? p.W / 2 : p.W;
+#pragma unroll
+  for (int j = 0; j < F; ++j) {
+    const int jr = q * F + j;
+    if (jr >= p.Co) break;  // warp-uniform
+    const int o = __ldg(p.perm + jr);
+    const float b = p.bias ? __ldg(p.bias + jr) : 0.f;
+    float v[PX];
+#pragma unroll
+    for (int k = 0; k < PX; ++k) v[k] = acc[j][k] + b;
+    if (p.flags & PP_ADD_SKIP) {
+      if (r < p.H) {
+        const float* sk = p.skip + (((size_t)n * p.Co + o) * p.H + r) * p.W;
+#pragma unroll
+        for (int k = 0; k < PX; ++k)
+          if (cb + k < p.W) v[k] += __ldg(sk + cb + k);
+      }
+    }
+    if (p.flags & PP_RELU) {
+#pragma unroll
+      for (int k = 0; k < PX; ++k) v[k] = fmaxf(v[k], 0.f);
+    }
+    if (pool) {
+      float u[PX];
+#pragma unroll
+      for (int k = 0; k < PX; ++k) u[k] = __shfl_down_sync(0xffffffffu, v[k], 1);
+      if ((ly & 1) == 0 && r < p.H) {
+        const int pr = r >> 1;
+        float* yo = p.y + (((size_t)n * p.Co + o) * Ho + pr) * Wo;
+#pragma unroll
+        for (int m = 0; m < PX / 2; ++m) {
+          const int pc = (cb >> 1) + m;
+          if (pc < Wo) yo[pc] = fmaxf(fmaxf(v[2 * m], v[2 * m + 1]), fmaxf(u[2 * m], u[2 * m + 1]));
+        }
+      }
+    } else if (r < p.H) {
+      float* yo = p.y + (((size_t)n * p.Co + o) * Ho + r) * Wo;
+      if (cb + PX <= p.W && (p.W & 3) == 0) {
+        reinterpret_cast<float4*>(yo + cb)[0] = make_float4(v[0], v[1], v[2], v[3]);
+        reinterpret_cast<float4*>(yo + cb)[1] = make_float4(v[4], v[5], v[6], v[7]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < PX; ++k)
+          if (cb + k < p.W) yo[cb + k] = v[k];
+      }
+    }
+  }
+}
+
+}  // namespace
+
+// ----------------------------------------------------------------------------
+// Host side: device layout of a layer and the launch.
+// ----------------------------------------------------------------------------
+
+struct pp_layer {
+  int Co = 0, Ci = 0;
+  int mode = MODE_GENERIC;
+  int G = 0, nch = 0;
+  int64_t nE = 0;
+  bool has_bias = false;
+  void* dmem = nullptr;  // one allocation holding every array below
+  size_t dbytes = 0;
+  int* cofs = nullptr;
+  uint32_t* code = nullptr;
+  float4* wts = nullptr;
+  int* perm = nullptr;
+  float* bias = nullptr;
+};
+
+struct pp_dense {
+  pp_layer base;
+};
+
+namespace {
+
+struct Entry {
+  int32_t ch;      // input channel
+  int32_t slot;    // filter slot in the warp's group
+  uint32_t payload;
+  float w[4];
+};
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Map each pattern of the set to its ring index, or -1 when the set is not a
+// subset of the ring set.
+bool ring_map(const uint8_t* taps, int P, std::vector<int>& map) {
+  map.assign(P, -1);
+  for (int p = 0; p < P; ++p) {
+    uint16_t m = ppc::tap_mask(taps + 4 * p);
+    for (int r = 0; r < 8; ++r) {
+      uint8_t rt[4];
+      for (int s = 0; s < 4; ++s) rt[s] = (uint8_t)ring_tap(r, s);
+      if (ppc::tap_mask(rt) == m) map[p] = r;
+    }
+    if (map[p] < 0) return false;
+  }
+  return true;
+}
+
+// Build the device layout from per-filter entry lists (filters already in
+// reordered order) and upload it.
+pp_status build_layer(pp_layer* L, int Co, int Ci, const std::vector<std::vector<Entry>>& per_filter,
+                      const std::vector<int32_t>& perm, const float* bias_reordered, cudaStream_t stream) {
+  L->Co = Co;
+  L->Ci = Ci;
+  L->G = (Co + F - 1) / F;
+  L->nch = (Ci + CC - 1) / CC;
+  L->has_bias = bias_reordered != nullptr;
+  std::vector<int> cofs((size_t)L->G * (L->nch + 1));
+  std::vector<uint32_t> code;
+  std::vector<float> wts;
+  for (int q = 0; q < L->G; ++q) {
+    std::vector<Entry> es;
+    for (int j = q * F; j < std::min(Co, (q + 1) * F); ++j)
+      for (Entry e : per_filter[j]) {
+        e.slot = j - q * F;
+        es.push_back(e);
+      }
+    std::stable_sort(es.begin(), es.end(), [](const Entry& a, const Entry& b) {
+      return a.ch != b.ch ? a.ch < b.ch : a.slot < b.slot;
+    });
+    size_t k = 0;
+    for (int c = 0; c <= L->nch; ++c) {
+      while (k < es.size() && es[k].ch < c * CC) ++k;
+      cofs[(size_t)q * (L->nch + 1) + c] = (int)(code.size() + k);
+    }
+    for (const Entry& e : es) {
+      code.push_back(e.payload | (uint32_t(e.slot) << 16) | (uint32_t(e.ch % CC) << 20));
+      for (int s = 0; s < 4; ++s) wts.push_back(e.w[s]);
+    }
+  }
+  L->nE = (int64_t)code.size();
+  if (L->nE > INT32_MAX) return PP_ERR_UNSUPPORTED;
+  size_t off_cofs = 0;
+  size_t off_code = align_up(off_cofs + cofs.size() * 4, 256);
+  size_t off_wts = align_up(off_code + code.size() * 4, 256);
+  size_t off_perm = align_up(off_wts + wts.size() * 4, 256);
+  size_t off_bias = align_up(off_perm + (size_t)Co * 4, 256);
+  size_t total = align_up(off_bias + (size_t)Co * 4, 256);
+  std::vector<unsigned char> host(total, 0);
+  std::memcpy(host.data() + off_cofs, cofs.data(), cofs.size() * 4);
+  if (!code.empty()) std::memcpy(host.data() + off_code, code.data(), code.size() * 4);
+  if (!wts.empty()) std::memcpy(host.data() + off_wts, wts.data(), wts.size() * 4);
+  std::memcpy(host.data() + off_perm, perm.data(), (size_t)Co * 4);
+  if (bias_reordered) std::memcpy(host.data() + off_bias, bias_reordered, (size_t)Co * 4);
+  void* d = nullptr;
+  if (cudaMalloc(&d, total) != cudaSuccess) {
+    cudaGetLastError();
+    return PP_ERR_OOM;
+  }
+  if (cudaMemcpyAsync(d, host.data(), total, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess) {
+    cudaFree(d);
+    return PP_ERR_CUDA;
+  }
+  unsigned char* b = static_cast<unsigned char*>(d);
+  L->dmem = d;
+  L->dbytes = total;
+  L->cofs = reinterpret_cast<int*>(b + off_cofs);
+  L->code = reinterpret_cast<uint32_t*>(b + off_code);
+  L->wts = reinterpret_cast<float4*>(b + off_wts);
+  L->perm = reinterpret_cast<int*>(b + off_perm);
+  L->bias = reinterpret_cast<float*>(b + off_bias);
+  return PP_OK;
+}
+
+pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip, int N, int H, int W, int flags,
+                 cudaStream_t stream) {
+  if (!L || !x || !y || N < 1 || H < 1 || W < 1) return PP_ERR_INVALID_ARG;
+  if (flags & ~(PP_ADD_SKIP | PP_RELU | PP_POOL2)) return PP_ERR_INVALID_ARG;
+  if ((flags & PP_ADD_SKIP) && !skip) return PP_ERR_INVALID_ARG;
+  if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
+  if (((uintptr_t)y & 15) || ((uintptr_t)x & 3)) return PP_ERR_INVALID_ARG;
+  const int tiles_y = (H + TH - 1) / TH, tiles_x = (W + TW - 1) / TW;
+  if ((int64_t)tiles_y * tiles_x > INT32_MAX || N > 65535) return PP_ERR_UNSUPPORTED;
+  ConvParams p;
+  p.x = x;
+  p.y = y;
+  p.skip = (flags & PP_ADD_SKIP) ? skip : nullptr;
+  p.cofs = L->cofs;
+  p.code = L->code;
+  p.wts = L->wts;
+  p.perm = L->perm;
+  p.bias = L->has_bias ? L->bias : nullptr;
+  p.N = N;
+  p.Ci = L->Ci;
+  p.Co = L->Co;
+  p.H = H;
+  p.W = W;
+  p.nch = L->nch;
+  p.G = L->G;
+  p.tiles_x = tiles_x;
+  p.flags = flags;
+  dim3 grid(tiles_y * tiles_x, (L->G + NWF - 1) / NWF, N);
+  if (grid.y > 65535) return PP_ERR_UNSUPPORTED;
+  if (L->mode == MODE_RING8)
+    ppconv_kernel<MODE_RING8><<<grid, NTHREADS, 0, stream>>>(p);
+  else
+    ppconv_kernel<MODE_GENERIC><<<grid, NTHREADS, 0, stream>>>(p);
+  return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, void* stream, pp_layer** out) {
+  if (!pk || !out) return PP_ERR_INVALID_ARG;
+  pp_layer* L = new (std::nothrow) pp_layer;
+  if (!L) return PP_ERR_OOM;
+  std::vector<int> rmap;
+  L->mode = ring_map(pk->taps.data(), pk->P, rmap) ? MODE_RING8 : MODE_GENERIC;
+  std::vector<std::vector<Entry>> per_filter(pk->Co);
+  std::vector<float> bias_r;
+  if (bias) bias_r.resize(pk->Co);
+  for (int j = 0; j < pk->Co; ++j) {
+    if (bias) bias_r[j] = bias[pk->perm[j]];
+    for (int32_t e = pk->kptr[j]; e < pk->kptr[j + 1]; ++e) {
+      Entry en;
+      en.ch = pk->kidx[e];
+      en.slot = 0;
+      const int p = pk->kpat[e];
+      if (L->mode == MODE_RING8) {
+        // Reorder the 4 weights from the pattern's ascending taps to the ring
+        // pattern's ascending taps (same set, so the same order).
+        en.payload = (uint32_t)rmap[p];
+      } else {
+        const uint8_t* t = &pk->taps[4 * p];
+        en.payload = t[0] | (t[1] << 4) | (t[2] << 8) | (t[3] << 12) | (3u << 28);
+      }
+      for (int s = 0; s < 4; ++s) en.w[s] = pk->kw[(size_t)e * 4 + s];
+      per_filter[j].push_back(en);
+    }
+  }
+  pp_status st = build_layer(L, pk->Co, pk->Ci, per_filter, pk->perm, bias ? bias_r.data() : nullptr,
+                             (cudaStream_t)stream);
+  if (st != PP_OK) {
+    delete L;
+    return st;
+  }
+  *out = L;
+  return PP_OK;
+}
+
+extern "C" pp_status pp_layer_info(const pp_layer* L, int* Co, int* Ci, int64_t* device_bytes) {
+  if (!L) return PP_ERR_INVALID_ARG;
+  if (Co) *Co = L->Co;
+  if (Ci) *Ci = L->Ci;
+  if (device_bytes) *device_bytes = (int64_t)L->dbytes;
+  return PP_OK;
+}
+
+extern "C" pp_status pp_conv_forward(const pp_layer* L, const float* x, float* y, const float* skip, int N, int H,
+                                     int W, int flags, void* stream) {
+  return launch(L, x, y, skip, N, H, W, flags, (cudaStream_t)stream);
+}
+
+extern "C" void pp_layer_destroy(pp_layer* L) {
+  if (!L) return;
+  if (L->dmem) cudaFree(L->dmem);
+  delete L;
+}
+
+extern "C" pp_status pp_dense_create(const float* w, const float* bias, int Co, int Ci, void* stream,
+                                     pp_dense** out) {
+  if (!w || !out || Co < 1 || Ci < 1) return PP_ERR_INVALID_ARG;
+  if ((int64_t)Co * Ci > (int64_t(1) << 26)) return PP_ERR_UNSUPPORTED;
+  pp_dense* D = new (std::nothrow) pp_dense;
+  if (!D) return PP_ERR_OOM;
+  D->base.mode = MODE_GENERIC;
+  // A dense kernel is three entries of the generic path: taps 0-3, 4-7 and 8.
+  std::vector<std::vector<Entry>> per_filter(Co);
+  std::vector<int32_t> perm(Co);
+  for (int o = 0; o < Co; ++o) {
+    perm[o] = o;
+    for (int i = 0; i < Ci; ++i) {
+      const float* k = w + ((size_t)o * Ci + i) * 9;
+      for (int part = 0; part < 3; ++part) {
+        Entry en;
+        en.ch = i;
+        en.slot = 0;
+        const int t0 = part * 4;
+        const int nt = part < 2 ? 4 : 1;
+        en.payload = 0;
+        for (int s = 0; s < nt; ++s) en.payload |= uint32_t(t0 + s) << (4 * s);
+        en.payload |= uint32_t(nt - 1) << 28;
+        for (int s = 0; s < 4; ++s) en.w[s] = s < nt ? k[t0 + s] : 0.f;
+        per_filter[o].push_back(en);
+      }
+    }
+  }
+  pp_status st = build_layer(&D->base, Co, Ci, per_filter, perm, bias, (cudaStream_t)stream);
+  if (st != PP_OK) {
+    delete D;
+    return st;
+  }
+  *out = D;
+  return PP_OK;
+}
+
+extern "C" pp_status pp_dense_forward(const pp_dense* D, const float* x, float* y, const float* skip, int N, int H,
+                                      int W, int flags, void* stream) {
+  if (!D) return PP_ERR_INVALID_ARG;
+  return launch(&D->base, x, y, skip, N, H, W, flags, (cudaStream_t)stream);
+}
+
+extern "C" pp_status pp_dense_info(const pp_dense* D, int* Co, int* Ci) {
+  if (!D) return PP_ERR_INVALID_ARG;
+  if (Co) *Co = D->base.Co;
+  if (Ci) *Ci = D->base.Ci;
+  return PP_OK;
+}
+
+extern "C" void pp_dense_destroy(pp_dense* D) {
+  if (!D) return;
+  if (D->base.dmem) cudaFree(D->base.dmem);
+  delete D;
+}

@@ -1,0 +1,147 @@
+"""The C-ABI library on the host (CPU only): it loads, exports every declared
+symbol, and its host packer matches the oracle bit for bit (Section 3 storage
+and reorder), including the validation errors of Section 2's invariants."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2004_11250_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def pp():
+    from paper_2004_11250_gb300 import build
+    build.build()
+    from paper_2004_11250_gb300 import ppconv
+    return ppconv
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "ppconv.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(pp_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(pp):
+    names = declared_symbols()
+    assert len(names) >= 20
+    for name in names:
+        assert hasattr(pp.lib, name), name
+
+
+def test_status_strings(pp):
+    assert pp.pp_status_string(0) == "PP_OK"
+    assert pp.pp_status_string(6) == "PP_ERR_UNSUPPORTED"
+    assert pp.pp_status_string(999) == "PP_ERR_UNKNOWN"
+    assert pp.pp_version() >= 100
+
+
+def layers_for_pack():
+    rng = np.random.default_rng(0)
+    out = [synth.small_random_layer(rng, 16, 16, P=8, keep=0.5),
+           synth.small_random_layer(rng, 64, 48, P=4, keep=0.2, ring=False),
+           synth.small_random_layer(rng, 33, 7, P=12, keep=0.9, ring=False),
+           synth.small_random_layer(rng, 5, 1, P=8, keep=1.0),
+           synth.small_random_layer(rng, 40, 40, P=8, keep=0.02),
+           synth.cfg0_single().ops[0].layer,
+           synth.cfg1_vgg16().ops[3].layer]
+    return out
+
+
+@pytest.mark.parametrize("idx", range(7))
+def test_pack_matches_oracle_bit_exact(pp, oracle_mod, idx):
+    L = layers_for_pack()[idx]
+    ref = oracle_mod.pack(L.w, L.mask, L.taps)
+    for ids in (None, L.pattern_ids):
+        pk = pp.pp_pack_layer(L.w, L.mask, L.taps, ids)
+        try:
+            a = pp.pp_packed_arrays(pk)
+            assert pp.pp_packed_info(pk) == (L.nk, L.Co, L.Ci, L.taps.shape[0])
+            assert (a["perm"] == ref.perm).all()
+            assert (a["kptr"] == ref.kptr).all()
+            assert (a["kidx"] == ref.kidx).all()
+            assert (a["kpat"] == ref.kpat).all()
+            assert (a["kw"].view(np.uint32) == ref.kw.view(np.uint32)).all()
+            assert (a["taps"] == L.taps).all()
+            w, m = pp.pp_unpack_layer(pk)
+            assert (m == L.mask).all()
+            assert (w.view(np.uint32) == L.w.view(np.uint32)).all()
+        finally:
+            pp.pp_packed_destroy(pk)
+
+
+def test_pack_hand_fixture(pp):
+    import json
+    g = json.load(open(os.path.join(ROOT, "tests", "golden", "hand_packed_layer.json")))
+    taps = np.array(g["taps"], np.uint8)
+    w = np.zeros((g["Co"], g["Ci"], 9), np.float32)
+    mask = np.zeros((g["Co"], g["Ci"]), np.uint8)
+    for o, i, p in g["kept"]:
+        mask[o, i] = 1
+        for t in taps[p]:
+            w[o, i, t] = 100 * o + 10 * i + t + 1
+    pk = pp.pp_pack_layer(w, mask, taps)
+    a = pp.pp_packed_arrays(pk)
+    pp.pp_packed_destroy(pk)
+    for k in ("perm", "kptr", "kidx", "kpat", "kw"):
+        assert a[k].tolist() == g[k], k
+
+
+def test_validation_errors_match_oracle(pp, oracle_mod):
+    rng = np.random.default_rng(3)
+    L = synth.small_random_layer(rng, 6, 5, P=8, keep=0.5)
+    cases = []
+    o, i = np.argwhere(L.mask == 0)[0]
+    w = L.w.copy()
+    w[o, i, 0] = 0.5
+    cases.append((w, L.mask, L.taps, None, pp.PP_ERR_PRUNED_NONZERO))
+    o, i = np.argwhere(L.mask == 1)[0]
+    w = L.w.copy()
+    w[o, i, :] = 1.0
+    cases.append((w, L.mask, L.taps, None, pp.PP_ERR_TAP_NOT_IN_PATTERN))
+    ids = L.pattern_ids.copy()
+    ids[o, i] = (ids[o, i] + 1) % 8
+    cases.append((L.w, L.mask, L.taps, ids, pp.PP_ERR_PATTERN_ID_MISMATCH))
+    for bad in ([[0, 1, 2, 9]], [[1, 0, 2, 4]], [[0, 1, 2, 4], [0, 1, 2, 4]]):
+        cases.append((np.zeros((1, 1, 9), np.float32), np.zeros((1, 1), np.uint8), np.array(bad, np.uint8), None,
+                      pp.PP_ERR_BAD_PATTERN_SET))
+    for w, m, t, ids, code in cases:
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_pack_layer(w, m, t, ids)
+        assert e.value.code == code
+        with pytest.raises(oracle_mod.OracleError) as e2:
+            oracle_mod.pack(w, m, t, ids)
+        assert e2.value.code == code  # the oracle uses the same numbering
+
+
+def test_pack_empty_and_invalid(pp):
+    taps = synth.ring8_patterns()
+    pk = pp.pp_pack_layer(np.zeros((3, 2, 9), np.float32), np.zeros((3, 2), np.uint8), taps)
+    a = pp.pp_packed_arrays(pk)
+    pp.pp_packed_destroy(pk)
+    assert a["perm"].tolist() == [0, 1, 2] and a["kptr"].tolist() == [0, 0, 0, 0] and a["kidx"].size == 0
+    with pytest.raises(pp.PPError) as e:
+        pp.pp_pack_layer(np.zeros((0, 2, 9), np.float32), np.zeros((0, 2), np.uint8), taps)
+    assert e.value.code == pp.PP_ERR_INVALID_ARG
+    # null handle arguments are rejected, not dereferenced
+    assert pp.lib.pp_packed_info(None, None, None, None, None) == pp.PP_ERR_INVALID_ARG
+    assert pp.lib.pp_conv_forward(None, None, None, None, 1, 1, 1, 0, None) == pp.PP_ERR_INVALID_ARG
+    assert pp.lib.pp_net_run(None, None, None, None) == pp.PP_ERR_INVALID_ARG
+    pp.pp_packed_destroy(None)
+    pp.pp_layer_destroy(None)
+    pp.pp_net_destroy(None)
+
+
+def test_net_shape_validation_host_only(pp):
+    """Network construction checks that need no device: bad shapes and flags."""
+    with pytest.raises(pp.PPError):
+        pp.pp_net_create(0, 1, 1, 1)
+    net = pp.pp_net_create(1, 3, 8, 8)
+    assert pp.pp_net_output_shape(net) == (1, 3, 8, 8)
+    with pytest.raises(pp.PPError):
+        pp.pp_net_finalize(net)  # no ops
+    pp.pp_net_destroy(net)

@@ -1,0 +1,218 @@
+"""GPU parity: the CUDA path, called through the C-ABI, against the fp64 oracle.
+
+Small layers are compared on every output; the five workloads at full size are
+compared layer by layer (each layer's oracle runs on the GPU's own input to that
+layer) on sampled outputs including borders and tile edges.  Bound:
+|gpu - oracle| <= 1e-5 * S per output (see tests/parity.py); integer-valued
+cases must be bit-exact.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2004_11250_gb300 import synth
+from parity import check_within, oracle_layer_full, oracle_layer_points, sample_points
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def pp():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2004_11250_gb300 import build
+    build.build()
+    from paper_2004_11250_gb300 import ppconv
+    return ppconv
+
+
+@pytest.fixture(scope="module")
+def runner(pp):
+    from paper_2004_11250_gb300 import runner
+    return runner
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def run_layer(pp, runner, layer, x, skip=None, relu=False, pool=False):
+    L = runner.DeviceLayer(layer)
+    try:
+        N, _, H, W = x.shape
+        Ho, Wo = (H // 2, W // 2) if pool else (H, W)
+        y = torch.full((N, layer.Co, Ho, Wo), float("nan"), device="cuda")
+        flags = (pp.PP_ADD_SKIP if skip is not None else 0) | (pp.PP_RELU if relu else 0) | (pp.PP_POOL2 if pool else 0)
+        L.forward(dev(x), y, None if skip is None else dev(skip), N, H, W, flags, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        return y.cpu().numpy()
+    finally:
+        L.close()
+
+
+SMALL = [
+    # N, Ci, Co, H, W, P, ring, keep
+    (1, 1, 1, 1, 1, 8, True, 1.0),
+    (1, 3, 5, 7, 9, 8, True, 0.6),
+    (2, 16, 16, 32, 32, 8, True, 0.5),
+    (1, 17, 33, 17, 33, 8, True, 0.3),
+    (2, 40, 20, 19, 40, 4, False, 0.35),
+    (1, 20, 40, 16, 16, 12, False, 0.5),
+    (1, 35, 18, 33, 18, 8, True, 1.0),
+    (3, 5, 7, 2, 3, 8, False, 0.9),
+    (1, 64, 64, 12, 44, 8, True, 0.2),
+]
+
+
+@pytest.mark.parametrize("case", SMALL)
+@pytest.mark.parametrize("flags", ["none", "relu", "skip_relu", "pool_relu"])
+def test_layer_parity_small(pp, runner, oracle_mod, case, flags):
+    N, Ci, Co, H, W, P, ring, keep = case
+    if flags == "pool_relu" and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(hash((case, flags)) % (2 ** 32))
+    L = synth.small_random_layer(rng, Co, Ci, P=P, keep=keep, ring=ring)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    relu = flags != "none"
+    pool = flags == "pool_relu"
+    g = run_layer(pp, runner, L, x, skip, relu, pool)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, relu, pool)
+    check_within(g, y, s, f"{case} {flags}")
+
+
+@pytest.mark.parametrize("ring", [True, False])
+def test_integer_layer_bit_exact(pp, runner, oracle_mod, ring):
+    """Small-integer weights and inputs: every partial sum is exact in fp32, so GPU == oracle bit for bit."""
+    rng = np.random.default_rng(5 if ring else 6)
+    taps = synth.ring8_patterns() if ring else synth.seeded_patterns(rng, 8)
+    L = synth.integer_layer(rng, 37, 29, taps, 0.5)
+    x = rng.integers(-8, 9, (2, 29, 21, 35)).astype(np.float32)
+    g = run_layer(pp, runner, L, x)
+    y, _ = oracle_layer_full(oracle_mod, L, x)
+    assert (g.astype(np.float64) == y).all()
+
+
+def test_all_pruned_layer_gives_bias(pp, runner, oracle_mod):
+    rng = np.random.default_rng(8)
+    L = synth.small_random_layer(rng, 20, 10, P=8, keep=0.0)
+    assert L.nk == 0
+    x = rng.uniform(-1, 1, (1, 10, 9, 9)).astype(np.float32)
+    g = run_layer(pp, runner, L, x)
+    assert (g == L.bias[None, :, None, None]).all()
+
+
+def test_dense_layers(pp, runner, oracle_mod):
+    rng = np.random.default_rng(12)
+    for Co, Ci, H, W, relu, skip in ((64, 1, 37, 50, True, False), (1, 64, 40, 33, False, True),
+                                     (7, 5, 16, 16, True, False)):
+        D = synth.make_dense_layer(rng, Co, Ci, synth.he_std(Ci), 0.01)
+        x = rng.uniform(0, 1, (1, Ci, H, W)).astype(np.float32)
+        sk = rng.uniform(0, 1, (1, Co, H, W)).astype(np.float32) if skip else None
+        g = run_layer(pp, runner, D, x, sk, relu)
+        y, s = oracle_layer_full(oracle_mod, D, x, sk, relu)
+        check_within(g, y, s, f"dense {Co}x{Ci}")
+
+
+def test_cfg0_full(pp, runner, oracle_mod):
+    net = synth.cfg0_single()
+    L = net.ops[0].layer
+    g = run_layer(pp, runner, L, net.x)
+    y, s = oracle_layer_full(oracle_mod, L, net.x)
+    check_within(g, y, s, "cfg0")
+
+
+def layerwise_check(pp, runner, oracle_mod, net, npts, seed=0, check_net=True):
+    """Run a network op by op on the GPU and check every op on sampled outputs against the oracle
+    evaluated on the GPU's own input to that op; then check the executor reproduces the op-by-op
+    result bit for bit (direct launches and CUDA-graph replay) and the host-buffer path too."""
+    rng = np.random.default_rng(seed)
+    dn = runner.DeviceNet(net, use_graph=True)
+    try:
+        x = dev(net.x)
+        acts = dn.run_layerwise(x)
+        torch.cuda.synchronize()
+        worst = 0.0
+        for k, op in enumerate(net.ops):
+            xin = acts[k].cpu().numpy()
+            out = acts[k + 1].cpu().numpy()
+            skip = acts[op.skip_from].cpu().numpy() if op.skip_from >= 0 else None
+            N, Co, Ho, Wo = out.shape
+            pts = sample_points(rng, N, Co, Ho, Wo, npts)
+            y, s = oracle_layer_points(oracle_mod, op.layer, xin, pts, skip, op.relu, op.pool)
+            worst = max(worst, check_within(out[tuple(pts.T)], y, s, f"{net.name} op {k}"))
+        if check_net:
+            final = acts[-1]
+            y1 = torch.empty_like(final)
+            dn.run(x, y1)
+            dn.run(x, y1)  # second call replays the captured graph
+            torch.cuda.synchronize()
+            assert torch.equal(y1, final)
+            xh = torch.from_numpy(net.x).pin_memory()
+            yh = torch.empty(final.shape, dtype=torch.float32).pin_memory()
+            dn.run_host(xh, yh)
+            assert torch.equal(yh, final.cpu())
+        return worst
+    finally:
+        dn.close()
+
+
+def test_cfg1_vgg16(pp, runner, oracle_mod):
+    assert layerwise_check(pp, runner, oracle_mod, synth.cfg1_vgg16(), 1500) < 1e-5
+
+
+def test_cfg2_style(pp, runner, oracle_mod):
+    assert layerwise_check(pp, runner, oracle_mod, synth.cfg2_style(), 1500) < 1e-5
+
+
+@pytest.mark.slow
+def test_cfg3_vdsr(pp, runner, oracle_mod):
+    assert layerwise_check(pp, runner, oracle_mod, synth.cfg3_vdsr(), 1000) < 1e-5
+
+
+def test_cfg3_small_full(pp, runner, oracle_mod):
+    """The VDSR-shaped stack on a small ragged image, every output of every op checked."""
+    net = synth.cfg3_vdsr(H=37, W=45)
+    dn = runner.DeviceNet(net, use_graph=False)
+    try:
+        acts = dn.run_layerwise(dev(net.x))
+        torch.cuda.synchronize()
+        for k, op in enumerate(net.ops):
+            skip = acts[op.skip_from].cpu().numpy() if op.skip_from >= 0 else None
+            y, s = oracle_layer_full(oracle_mod, op.layer, acts[k].cpu().numpy(), skip, op.relu, op.pool)
+            check_within(acts[k + 1].cpu().numpy(), y, s, f"vdsr small op {k}")
+    finally:
+        dn.close()
+
+
+@pytest.mark.parametrize("point", synth.cfg4_points())
+def test_cfg4_sweep_point(pp, runner, oracle_mod, point):
+    C, P, keep = point
+    net = synth.cfg4_point(C, P, keep)
+    L = net.ops[0].layer
+    g = run_layer(pp, runner, L, net.x)
+    rng = np.random.default_rng(C + P + int(keep * 100))
+    pts = sample_points(rng, *g.shape, 400)
+    y, s = oracle_layer_points(oracle_mod, L, net.x, pts)
+    check_within(g[tuple(pts.T)], y, s, f"sweep {point}")
+
+
+def test_bad_arguments_rejected(pp, runner):
+    rng = np.random.default_rng(1)
+    L = runner.DeviceLayer(synth.small_random_layer(rng, 4, 4))
+    x = torch.zeros((1, 4, 5, 5), device="cuda")
+    y = torch.zeros((1, 4, 5, 5), device="cuda")
+    try:
+        with pytest.raises(pp.PPError) as e:
+            L.forward(x, y, None, 1, 5, 5, pp.PP_POOL2, None)
+        assert e.value.code == pp.PP_ERR_UNSUPPORTED
+        with pytest.raises(pp.PPError) as e:
+            L.forward(x, y, None, 1, 5, 5, pp.PP_ADD_SKIP, None)
+        assert e.value.code == pp.PP_ERR_INVALID_ARG
+        with pytest.raises(pp.PPError) as e:
+            L.forward(x, y, None, 1, 5, 5, 64, None)
+        assert e.value.code == pp.PP_ERR_INVALID_ARG
+        with pytest.raises(pp.PPError) as e:
+            L.forward(x, y, None, 0, 5, 5, 0, None)
+        assert e.value.code == pp.PP_ERR_INVALID_ARG
+    finally:
+        L.close()
