@@ -12,7 +12,13 @@
 //     accumulators are acc[16][8] registers, indexed only by compile-time
 //     constants.
 //   * Input channels are staged 16 at a time into shared memory (tile + 1-pixel
-//     halo, zero padding) with cp.async, double buffered.
+//     halo, zero padding) with cp.async, double buffered; each warp stages the
+//     entries of its filter group for the same channels next to them, so the
+//     entry stream is read from shared memory one entry ahead of its use.
+//   * Small grids (late VGG layers) split the input channels over the CTAs of
+//     a thread-block cluster; the partial accumulators are summed through
+//     distributed shared memory in a fixed rank order (deterministic) and the
+//     epilogue of each slot runs on one CTA of the cluster.
 //   * Per input channel a lane loads its 3x10 input window once into
 //     registers and reuses it for every kept kernel of that channel in its
 //     filter group: this reuse across filters is what keeps the FMA pipe fed
@@ -28,6 +34,7 @@
 //   * Epilogue: bias, optional residual add, ReLU, optional 2x2 max pool (the
 //     partner row comes from the neighbouring lane by shuffle), store to the
 //     filter's original channel.
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -49,8 +56,18 @@ constexpr int SROWS = TH + 2;
 constexpr int SCOLS = TW + 2;
 constexpr int SSTRIDE = 20;      // row stride (floats): 16B aligned, conflict-free LDS.128 per 8-lane phase
 constexpr int SCH = SROWS * SSTRIDE;
-constexpr int STAGE = CC * SCH;
+constexpr int STAGE_IN = CC * SCH;           // input floats per stage
+constexpr int EMAX = F * CC;                 // most entries a warp can have per stage
 constexpr int NTHREADS = 32 * NWF;
+// Stage layout in bytes: [weights NWF][EMAX] float4 | input [CC][SROWS][SSTRIDE] | codes [NWF][EMAX] u32
+constexpr int OFF_WTS = 0;
+constexpr int OFF_IN = OFF_WTS + NWF * EMAX * 16;
+constexpr int OFF_CODE = OFF_IN + STAGE_IN * 4;
+constexpr int STAGE_BYTES = OFF_CODE + NWF * EMAX * 4;
+constexpr int SMEM_BYTES = 2 * STAGE_BYTES;
+constexpr int RED_BYTES = NWF * F * PX * 32 * 4;  // split-K partials of one CTA
+static_assert(RED_BYTES <= SMEM_BYTES, "split-K partials must fit in the stage buffers");
+constexpr int MAX_SPLIT = 8;
 
 enum Mode { MODE_RING8 = 0, MODE_GENERIC = 1 };
 
@@ -81,6 +98,9 @@ struct ConvParams {
   int nch, G;
   int tiles_x;
   int flags;
+  int cc;      // input channels per stage (<= CC; entries per warp and stage stay <= EMAX)
+  int ksplit;  // CTAs of a cluster sharing one output tile (split over input chunks)
+  int cpk;     // input chunks per split
 };
 
 // Entry code layout: bits 0..15 pattern payload (MODE_RING8: ring index;
@@ -109,12 +129,17 @@ __device__ __forceinline__ void cp_async4(float* sdst, const float* gsrc, bool v
   int n = valid ? 4 : 0;
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(saddr), "l"(gsrc), "r"(n));
 }
+__device__ __forceinline__ void cp_async16(void* sdst, const void* gsrc) {
+  unsigned saddr = (unsigned)__cvta_generic_to_shared(sdst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(saddr), "l"(gsrc));
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
 
-// Stage channels [i0, i0 + nvalid) of image n, rows r0-1..r0+TH, cols c0-1..c0+TW.
-__device__ __forceinline__ void stage_chunk(float* s, const ConvParams& p, int n, int i0, int nvalid, int r0,
+// Stage input channels [i0, i0 + nvalid) of image n, rows r0-1..r0+TH, cols
+// c0-1..c0+TW, into `s` (zero outside the image), one 4-byte cp.async each.
+__device__ __forceinline__ void stage_input(float* s, const ConvParams& p, int n, int i0, int nvalid, int r0,
                                             int c0) {
   const int total = nvalid * SROWS * SCOLS;
   const float* xb = p.x + ((size_t)n * p.Ci + i0) * p.H * p.W;
@@ -127,6 +152,18 @@ __device__ __forceinline__ void stage_chunk(float* s, const ConvParams& p, int n
     const bool ok = (unsigned)r < (unsigned)p.H && (unsigned)c < (unsigned)p.W;
     const float* src = ok ? xb + ((size_t)ch * p.H + r) * p.W + c : p.x;
     cp_async4(s + ch * SCH + sr * SSTRIDE + sc, src, ok);
+  }
+}
+
+// Stage the entries [e0, e1) of this warp's filter group (at most EMAX) into
+// the warp's own slice of the stage.
+__device__ __forceinline__ void stage_entries(unsigned char* stage, const ConvParams& p, int warp, int lane, int e0,
+                                              int e1) {
+  float4* sw = reinterpret_cast<float4*>(stage + OFF_WTS) + warp * EMAX;
+  uint32_t* sc = reinterpret_cast<uint32_t*>(stage + OFF_CODE) + warp * EMAX;
+  for (int e = e0 + lane; e < e1; e += 32) {
+    cp_async16(sw + (e - e0), p.wts + e);
+    cp_async4(reinterpret_cast<float*>(sc + (e - e0)), reinterpret_cast<const float*>(p.code + e), true);
   }
 }
 
@@ -176,9 +213,58 @@ __device__ __forceinline__ void dispatch(float (&acc)[F][PX], const float (&win)
   }
 }
 
-template <int MODE>
+// Epilogue of one filter slot: bias, +skip, ReLU, 2x2 max pool, store at the
+// filter's original channel.  Must be called by all 32 lanes (the pool reads
+// the partner row from the next lane).
+__device__ __forceinline__ void epilogue_slot(const ConvParams& p, int n, int q, int j, float (&v)[PX], int r,
+                                              int cb, int ly) {
+  const int jr = q * F + j;
+  const int o = __ldg(p.perm + jr);
+  const float b = p.bias ? __ldg(p.bias + jr) : 0.f;
+  const bool pool = p.flags & PP_POOL2;
+  const int Ho = pool ? p.H / 2 : p.H, Wo = pool ? p.W / 2 : p.W;
+#pragma unroll
+  for (int k = 0; k < PX; ++k) v[k] += b;
+  if (p.flags & PP_ADD_SKIP) {
+    if (r < p.H) {
+      const float* sk = p.skip + (((size_t)n * p.Co + o) * p.H + r) * p.W;
+#pragma unroll
+      for (int k = 0; k < PX; ++k)
+        if (cb + k < p.W) v[k] += __ldg(sk + cb + k);
+    }
+  }
+  if (p.flags & PP_RELU) {
+#pragma unroll
+    for (int k = 0; k < PX; ++k) v[k] = fmaxf(v[k], 0.f);
+  }
+  if (pool) {
+    float u[PX];
+#pragma unroll
+    for (int k = 0; k < PX; ++k) u[k] = __shfl_down_sync(0xffffffffu, v[k], 1);
+    if ((ly & 1) == 0 && r < p.H) {
+      float* yo = p.y + (((size_t)n * p.Co + o) * Ho + (r >> 1)) * Wo;
+#pragma unroll
+      for (int m = 0; m < PX / 2; ++m) {
+        const int pc = (cb >> 1) + m;
+        if (pc < Wo) yo[pc] = fmaxf(fmaxf(v[2 * m], v[2 * m + 1]), fmaxf(u[2 * m], u[2 * m + 1]));
+      }
+    }
+  } else if (r < p.H) {
+    float* yo = p.y + (((size_t)n * p.Co + o) * Ho + r) * Wo;
+    if (cb + PX <= p.W && (p.W & 3) == 0) {
+      reinterpret_cast<float4*>(yo + cb)[0] = make_float4(v[0], v[1], v[2], v[3]);
+      reinterpret_cast<float4*>(yo + cb)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < PX; ++k)
+        if (cb + k < p.W) yo[cb + k] = v[k];
+    }
+  }
+}
+
+template <int MODE, bool SPLIT>
 __global__ void __launch_bounds__(NTHREADS, 2) ppconv_kernel(const ConvParams p) {
-  __shared__ __align__(16) float smem[2 * STAGE];
+  extern __shared__ __align__(16) unsigned char smem[];
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -187,7 +273,8 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_kernel(const ConvParams p)
   const int tile = blockIdx.x;
   const int ty = tile / p.tiles_x, tx = tile - ty * p.tiles_x;
   const int r0 = ty * TH, c0 = tx * TW;
-  const int n = blockIdx.z;
+  const int n = SPLIT ? blockIdx.z / p.ksplit : blockIdx.z;
+  const int ks = SPLIT ? blockIdx.z - n * p.ksplit : 0;
   const int q = blockIdx.y * NWF + warp;  // filter group of this warp
   const bool active = q < p.G;
 
@@ -198,30 +285,46 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_kernel(const ConvParams p)
     for (int k = 0; k < PX; ++k) acc[j][k] = 0.f;
 
   const int* cofs = p.cofs + (size_t)(active ? q : 0) * (p.nch + 1);
+  const int cbeg = ks * p.cpk;
+  const int cend = min(p.nch, cbeg + p.cpk);
 
-  stage_chunk(smem, p, n, 0, min(CC, p.Ci), r0, c0);
-  cp_async_commit();
-  for (int c = 0; c < p.nch; ++c) {
-    if (c + 1 < p.nch) {
-      stage_chunk(smem + ((c + 1) & 1) * STAGE, p, n, (c + 1) * CC, min(CC, p.Ci - (c + 1) * CC), r0, c0);
-      cp_async_commit();
+  auto issue = [&](int c) {
+    unsigned char* st = smem + (c & 1) * STAGE_BYTES;
+    stage_input(reinterpret_cast<float*>(st + OFF_IN), p, n, c * p.cc, min(p.cc, p.Ci - c * p.cc), r0, c0);
+    if (active) stage_entries(st, p, warp, lane, __ldg(cofs + c), __ldg(cofs + c + 1));
+    cp_async_commit();
+  };
+
+  if (cbeg < cend) issue(cbeg);
+  for (int c = cbeg; c < cend; ++c) {
+    if (c + 1 < cend) {
+      issue(c + 1);
       cp_async_wait<1>();
     } else {
       cp_async_wait<0>();
     }
     __syncthreads();
     if (active) {
-      const float* sb = smem + (c & 1) * STAGE + ly * SSTRIDE + lx * PX;
-      const int e0 = __ldg(cofs + c), e1 = __ldg(cofs + c + 1);
+      const unsigned char* st = smem + (c & 1) * STAGE_BYTES;
+      const float* sb = reinterpret_cast<const float*>(st + OFF_IN) + ly * SSTRIDE + lx * PX;
+      const float4* sw = reinterpret_cast<const float4*>(st + OFF_WTS) + warp * EMAX;
+      const uint32_t* sc = reinterpret_cast<const uint32_t*>(st + OFF_CODE) + warp * EMAX;
+      const int ne = __ldg(cofs + c + 1) - __ldg(cofs + c);
       int cur = -1;
       float win[3][PX + 2];
 #pragma unroll
       for (int a = 0; a < 3; ++a)
 #pragma unroll
         for (int b = 0; b < PX + 2; ++b) win[a][b] = 0.f;
-      for (int e = e0; e < e1; ++e) {
-        const uint32_t code = __ldg(p.code + e);
-        const float4 w = __ldg(p.wts + e);
+      uint32_t code_n = ne > 0 ? sc[0] : 0u;
+      float4 w_n = ne > 0 ? sw[0] : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int e = 0; e < ne; ++e) {
+        const uint32_t code = code_n;
+        const float4 w = w_n;
+        if (e + 1 < ne) {
+          code_n = sc[e + 1];
+          w_n = sw[e + 1];
+        }
         const int ch = code_ch(code);
         if (ch != cur) {
           cur = ch;
@@ -241,58 +344,44 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_kernel(const ConvParams p)
     }
     __syncthreads();
   }
-  if (!active) return;
 
-  // Epilogue: bias, +skip, ReLU, 2x2 max pool, store at the original channel.
   const int r = r0 + ly;
   const int cb = c0 + lx * PX;
-  const bool pool = p.flags & PP_POOL2;
-  const int Ho = pool ? p.H / 2 : p.H, Wo = pool ? p.W / 2 : p.W;
+  if constexpr (!SPLIT) {
+    if (!active) return;
 #pragma unroll
-  for (int j = 0; j < F; ++j) {
-    const int jr = q * F + j;
-    if (jr >= p.Co) break;  // warp-uniform
-    const int o = __ldg(p.perm + jr);
-    const float b = p.bias ? __ldg(p.bias + jr) : 0.f;
-    float v[PX];
-#pragma unroll
-    for (int k = 0; k < PX; ++k) v[k] = acc[j][k] + b;
-    if (p.flags & PP_ADD_SKIP) {
-      if (r < p.H) {
-        const float* sk = p.skip + (((size_t)n * p.Co + o) * p.H + r) * p.W;
-#pragma unroll
-        for (int k = 0; k < PX; ++k)
-          if (cb + k < p.W) v[k] += __ldg(sk + cb + k);
-      }
+    for (int j = 0; j < F; ++j) {
+      if (q * F + j >= p.Co) break;  // warp-uniform
+      epilogue_slot(p, n, q, j, acc[j], r, cb, ly);
     }
-    if (p.flags & PP_RELU) {
+  } else {
+    // Split over input chunks: publish the partial sums in this CTA's shared
+    // memory, then every CTA of the cluster reduces the slots j with
+    // j % ksplit == its rank, reading all ranks in order 0..ksplit-1.
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    float* red = reinterpret_cast<float*>(smem);
 #pragma unroll
-      for (int k = 0; k < PX; ++k) v[k] = fmaxf(v[k], 0.f);
-    }
-    if (pool) {
-      float u[PX];
+    for (int j = 0; j < F; ++j)
 #pragma unroll
-      for (int k = 0; k < PX; ++k) u[k] = __shfl_down_sync(0xffffffffu, v[k], 1);
-      if ((ly & 1) == 0 && r < p.H) {
-        const int pr = r >> 1;
-        float* yo = p.y + (((size_t)n * p.Co + o) * Ho + pr) * Wo;
+      for (int k = 0; k < PX; ++k) red[((warp * F + j) * PX + k) * 32 + lane] = acc[j][k];
+    cluster.sync();
+    const int rank = (int)cluster.block_rank();
+    if (active) {
+      for (int j = rank; j < F; j += p.ksplit) {
+        if (q * F + j >= p.Co) break;  // warp-uniform
+        float v[PX];
 #pragma unroll
-        for (int m = 0; m < PX / 2; ++m) {
-          const int pc = (cb >> 1) + m;
-          if (pc < Wo) yo[pc] = fmaxf(fmaxf(v[2 * m], v[2 * m + 1]), fmaxf(u[2 * m], u[2 * m + 1]));
+        for (int k = 0; k < PX; ++k) v[k] = 0.f;
+        for (int s2 = 0; s2 < p.ksplit; ++s2) {
+          const float* rem = cluster.map_shared_rank(red, s2);
+#pragma unroll
+          for (int k = 0; k < PX; ++k) v[k] += rem[((warp * F + j) * PX + k) * 32 + lane];
         }
-      }
-    } else if (r < p.H) {
-      float* yo = p.y + (((size_t)n * p.Co + o) * Ho + r) * Wo;
-      if (cb + PX <= p.W && (p.W & 3) == 0) {
-        reinterpret_cast<float4*>(yo + cb)[0] = make_float4(v[0], v[1], v[2], v[3]);
-        reinterpret_cast<float4*>(yo + cb)[1] = make_float4(v[4], v[5], v[6], v[7]);
-      } else {
-#pragma unroll
-        for (int k = 0; k < PX; ++k)
-          if (cb + k < p.W) yo[cb + k] = v[k];
+        epilogue_slot(p, n, q, j, v, r, cb, ly);
       }
     }
+    cluster.sync();  // keep every CTA's shared memory alive until all reads are done
   }
 }
 
@@ -306,6 +395,7 @@ struct pp_layer {
   int Co = 0, Ci = 0;
   int mode = MODE_GENERIC;
   int G = 0, nch = 0;
+  int cc = CC;  // input channels per stage
   int64_t nE = 0;
   bool has_bias = false;
   void* dmem = nullptr;  // one allocation holding every array below
@@ -350,12 +440,13 @@ bool ring_map(const uint8_t* taps, int P, std::vector<int>& map) {
 
 // Build the device layout from per-filter entry lists (filters already in
 // reordered order) and upload it.
-pp_status build_layer(pp_layer* L, int Co, int Ci, const std::vector<std::vector<Entry>>& per_filter,
+pp_status build_layer(pp_layer* L, int Co, int Ci, int cc, const std::vector<std::vector<Entry>>& per_filter,
                       const std::vector<int32_t>& perm, const float* bias_reordered, cudaStream_t stream) {
   L->Co = Co;
   L->Ci = Ci;
+  L->cc = cc;
   L->G = (Co + F - 1) / F;
-  L->nch = (Ci + CC - 1) / CC;
+  L->nch = (Ci + cc - 1) / cc;
   L->has_bias = bias_reordered != nullptr;
   std::vector<int> cofs((size_t)L->G * (L->nch + 1));
   std::vector<uint32_t> code;
@@ -372,11 +463,14 @@ pp_status build_layer(pp_layer* L, int Co, int Ci, const std::vector<std::vector
     });
     size_t k = 0;
     for (int c = 0; c <= L->nch; ++c) {
-      while (k < es.size() && es[k].ch < c * CC) ++k;
+      while (k < es.size() && es[k].ch < c * cc) ++k;
       cofs[(size_t)q * (L->nch + 1) + c] = (int)(code.size() + k);
     }
+    for (int c = 0; c < L->nch; ++c)  // the kernel stages at most EMAX entries per warp and chunk
+      if (cofs[(size_t)q * (L->nch + 1) + c + 1] - cofs[(size_t)q * (L->nch + 1) + c] > EMAX)
+        return PP_ERR_UNSUPPORTED;
     for (const Entry& e : es) {
-      code.push_back(e.payload | (uint32_t(e.slot) << 16) | (uint32_t(e.ch % CC) << 20));
+      code.push_back(e.payload | (uint32_t(e.slot) << 16) | (uint32_t(e.ch % cc) << 20));
       for (int s = 0; s < 4; ++s) wts.push_back(e.w[s]);
     }
   }
@@ -415,6 +509,37 @@ pp_status build_layer(pp_layer* L, int Co, int Ci, const std::vector<std::vector
   return PP_OK;
 }
 
+template <int MODE, bool SPLIT>
+cudaError_t set_attributes() {
+  cudaError_t e = cudaFuncSetAttribute(ppconv_kernel<MODE, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       SMEM_BYTES);
+  return e;
+}
+
+// Once per process and device: allow the kernels' dynamic shared memory.
+cudaError_t prepare_kernels() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  static bool done[64] = {};
+  if (dev < 64 && done[dev]) return cudaSuccess;
+  if ((e = set_attributes<MODE_RING8, false>()) != cudaSuccess) return e;
+  if ((e = set_attributes<MODE_RING8, true>()) != cudaSuccess) return e;
+  if ((e = set_attributes<MODE_GENERIC, false>()) != cudaSuccess) return e;
+  if ((e = set_attributes<MODE_GENERIC, true>()) != cudaSuccess) return e;
+  if (dev < 64) done[dev] = true;
+  return cudaSuccess;
+}
+
+// Number of CTAs sharing one output tile: split the input chunks over a
+// cluster when the grid alone would leave SMs idle (two CTAs fit per SM).
+int choose_split(int64_t base_ctas, int nch) {
+  int sms = 152;
+  int ks = 1;
+  while (ks < MAX_SPLIT && ks * 2 <= nch && base_ctas * ks < 2 * sms) ks *= 2;
+  return ks;
+}
+
 pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip, int N, int H, int W, int flags,
                  cudaStream_t stream) {
   if (!L || !x || !y || N < 1 || H < 1 || W < 1) return PP_ERR_INVALID_ARG;
@@ -423,7 +548,7 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   if (((uintptr_t)y & 15) || ((uintptr_t)x & 3)) return PP_ERR_INVALID_ARG;
   const int tiles_y = (H + TH - 1) / TH, tiles_x = (W + TW - 1) / TW;
-  if ((int64_t)tiles_y * tiles_x > INT32_MAX || N > 65535) return PP_ERR_UNSUPPORTED;
+  if ((int64_t)tiles_y * tiles_x > INT32_MAX) return PP_ERR_UNSUPPORTED;
   ConvParams p;
   p.x = x;
   p.y = y;
@@ -439,22 +564,49 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   p.H = H;
   p.W = W;
   p.nch = L->nch;
+  p.cc = L->cc;
   p.G = L->G;
   p.tiles_x = tiles_x;
   p.flags = flags;
-  dim3 grid(tiles_y * tiles_x, (L->G + NWF - 1) / NWF, N);
-  if (grid.y > 65535) return PP_ERR_UNSUPPORTED;
-  if (L->mode == MODE_RING8)
-    ppconv_kernel<MODE_RING8><<<grid, NTHREADS, 0, stream>>>(p);
-  else
-    ppconv_kernel<MODE_GENERIC><<<grid, NTHREADS, 0, stream>>>(p);
-  return cudaGetLastError() == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+  const int cgroups = (L->G + NWF - 1) / NWF;
+  const int64_t base = (int64_t)tiles_y * tiles_x * cgroups * N;
+  const int ks = choose_split(base, L->nch);
+  p.ksplit = ks;
+  p.cpk = (L->nch + ks - 1) / ks;
+  if ((int64_t)N * ks > 65535 || cgroups > 65535) return PP_ERR_UNSUPPORTED;
+  if (prepare_kernels() != cudaSuccess) return PP_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(tiles_y * tiles_x, cgroups, N * ks);
+  cfg.blockDim = dim3(NTHREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  cudaError_t e;
+  if (ks > 1) {
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = ks;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = L->mode == MODE_RING8 ? cudaLaunchKernelEx(&cfg, ppconv_kernel<MODE_RING8, true>, p)
+                              : cudaLaunchKernelEx(&cfg, ppconv_kernel<MODE_GENERIC, true>, p);
+  } else {
+    e = L->mode == MODE_RING8 ? cudaLaunchKernelEx(&cfg, ppconv_kernel<MODE_RING8, false>, p)
+                              : cudaLaunchKernelEx(&cfg, ppconv_kernel<MODE_GENERIC, false>, p);
+  }
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return PP_ERR_CUDA;
+  }
+  return PP_OK;
 }
 
 }  // namespace
 
 extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, void* stream, pp_layer** out) {
   if (!pk || !out) return PP_ERR_INVALID_ARG;
+  if (prepare_kernels() != cudaSuccess) return PP_ERR_CUDA;  // outside any stream capture
   pp_layer* L = new (std::nothrow) pp_layer;
   if (!L) return PP_ERR_OOM;
   std::vector<int> rmap;
@@ -481,7 +633,7 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
       per_filter[j].push_back(en);
     }
   }
-  pp_status st = build_layer(L, pk->Co, pk->Ci, per_filter, pk->perm, bias ? bias_r.data() : nullptr,
+  pp_status st = build_layer(L, pk->Co, pk->Ci, CC, per_filter, pk->perm, bias ? bias_r.data() : nullptr,
                              (cudaStream_t)stream);
   if (st != PP_OK) {
     delete L;
@@ -514,6 +666,7 @@ extern "C" pp_status pp_dense_create(const float* w, const float* bias, int Co, 
                                      pp_dense** out) {
   if (!w || !out || Co < 1 || Ci < 1) return PP_ERR_INVALID_ARG;
   if ((int64_t)Co * Ci > (int64_t(1) << 26)) return PP_ERR_UNSUPPORTED;
+  if (prepare_kernels() != cudaSuccess) return PP_ERR_CUDA;
   pp_dense* D = new (std::nothrow) pp_dense;
   if (!D) return PP_ERR_OOM;
   D->base.mode = MODE_GENERIC;
@@ -538,7 +691,8 @@ extern "C" pp_status pp_dense_create(const float* w, const float* bias, int Co, 
       }
     }
   }
-  pp_status st = build_layer(&D->base, Co, Ci, per_filter, perm, bias, (cudaStream_t)stream);
+  // three entries per kernel: 5 channels per stage keep a warp's stage at <= EMAX entries
+  pp_status st = build_layer(&D->base, Co, Ci, 5, per_filter, perm, bias, (cudaStream_t)stream);
   if (st != PP_OK) {
     delete D;
     return st;
