@@ -144,6 +144,18 @@ pp_status pp_layer_info(const pp_layer* layer, int* Co, int* Ci, int64_t* device
 pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H, int W,
                           int flags, void* stream);
 
+/* Which kernel pp_conv_forward runs for a layer.  PP_KERNEL_AUTO picks the
+ * tensor-memory kernel when every pattern is a ring pattern (the centre tap
+ * plus 3 consecutive of its 8 neighbours) and the register kernel otherwise.
+ * Setting PP_KERNEL_TMEM on a layer whose patterns are not all ring patterns
+ * returns PP_ERR_UNSUPPORTED.  Both kernels compute the same convolution. */
+#define PP_KERNEL_AUTO 0
+#define PP_KERNEL_TMEM 1
+#define PP_KERNEL_REGISTER 2
+pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
+/* The kernel that pp_conv_forward will run (PP_KERNEL_TMEM or PP_KERNEL_REGISTER). */
+pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
+
 void pp_layer_destroy(pp_layer* layer);
 
 /* ------------------------------------------------------------------------

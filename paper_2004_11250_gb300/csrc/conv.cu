@@ -394,6 +394,9 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_kernel(const ConvParams p)
 struct pp_layer {
   int Co = 0, Ci = 0;
   int mode = MODE_GENERIC;
+  bool tm_ok = false;    // ring-set layer: the tensor-memory kernel can run it
+  bool use_tm = false;
+  ppc::TmLayout tm;
   int G = 0, nch = 0;
   int cc = CC;  // input channels per stage
   int64_t nE = 0;
@@ -547,6 +550,14 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   if ((flags & PP_ADD_SKIP) && !skip) return PP_ERR_INVALID_ARG;
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   if (((uintptr_t)y & 15) || ((uintptr_t)x & 3)) return PP_ERR_INVALID_ARG;
+  if (L->use_tm) {
+    ppc::LayerMeta M;
+    M.Co = L->Co;
+    M.Ci = L->Ci;
+    M.perm = L->perm;
+    M.bias = L->has_bias ? L->bias : nullptr;
+    return ppc::tm_launch(L->tm, M, x, y, skip, N, H, W, flags, stream);
+  }
   const int tiles_y = (H + TH - 1) / TH, tiles_x = (W + TW - 1) / TW;
   if ((int64_t)tiles_y * tiles_x > INT32_MAX) return PP_ERR_UNSUPPORTED;
   ConvParams p;
@@ -635,11 +646,37 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
   }
   pp_status st = build_layer(L, pk->Co, pk->Ci, CC, per_filter, pk->perm, bias ? bias_r.data() : nullptr,
                              (cudaStream_t)stream);
+  if (st == PP_OK && L->mode == MODE_RING8) {
+    st = ppc::tm_prepare();
+    if (st == PP_OK) st = ppc::tm_build(&L->tm, pk, rmap, (cudaStream_t)stream);
+    L->tm_ok = st == PP_OK;
+    L->use_tm = L->tm_ok;
+  }
   if (st != PP_OK) {
-    delete L;
+    pp_layer_destroy(L);
     return st;
   }
   *out = L;
+  return PP_OK;
+}
+
+extern "C" pp_status pp_layer_set_kernel(pp_layer* L, int kernel) {
+  if (!L) return PP_ERR_INVALID_ARG;
+  if (kernel == PP_KERNEL_AUTO || kernel == PP_KERNEL_TMEM) {
+    if (kernel == PP_KERNEL_TMEM && !L->tm_ok) return PP_ERR_UNSUPPORTED;
+    L->use_tm = L->tm_ok;
+    return PP_OK;
+  }
+  if (kernel == PP_KERNEL_REGISTER) {
+    L->use_tm = false;
+    return PP_OK;
+  }
+  return PP_ERR_INVALID_ARG;
+}
+
+extern "C" pp_status pp_layer_kernel(const pp_layer* L, int* kernel) {
+  if (!L || !kernel) return PP_ERR_INVALID_ARG;
+  *kernel = L->use_tm ? PP_KERNEL_TMEM : PP_KERNEL_REGISTER;
   return PP_OK;
 }
 
@@ -647,7 +684,7 @@ extern "C" pp_status pp_layer_info(const pp_layer* L, int* Co, int* Ci, int64_t*
   if (!L) return PP_ERR_INVALID_ARG;
   if (Co) *Co = L->Co;
   if (Ci) *Ci = L->Ci;
-  if (device_bytes) *device_bytes = (int64_t)L->dbytes;
+  if (device_bytes) *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes);
   return PP_OK;
 }
 
@@ -659,6 +696,7 @@ extern "C" pp_status pp_conv_forward(const pp_layer* L, const float* x, float* y
 extern "C" void pp_layer_destroy(pp_layer* L) {
   if (!L) return;
   if (L->dmem) cudaFree(L->dmem);
+  if (L->tm.dmem) cudaFree(L->tm.dmem);
   delete L;
 }
 

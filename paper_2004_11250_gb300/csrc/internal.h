@@ -1,6 +1,8 @@
 // Internal declarations shared by the library's translation units.
 #pragma once
 
+#include <cuda_runtime.h>
+
 #include <cstdint>
 #include <vector>
 
@@ -26,9 +28,31 @@ constexpr int kSlots = 16;
 // Input channels staged in shared memory per pipeline step.
 constexpr int kChunk = 16;
 
-// Tap-set identifiers.  A pattern's taps are encoded as a 9-bit mask; the
-// kernels specialise on the fixed ring set of 8 centre-based patterns and fall
-// back to a per-tap dispatch for any other set.
+// A pattern's taps as a 9-bit mask.
 uint16_t tap_mask(const uint8_t* taps4);
+
+// Device-side description shared by every kernel of a layer.
+struct LayerMeta {
+  int Co = 0, Ci = 0;
+  const int* perm = nullptr;    // [Co] original channel of reordered filter j
+  const float* bias = nullptr;  // [Co] bias in reordered order, or null
+};
+
+// Entry blobs of the tensor-memory kernel (conv_tm.cu).
+struct TmLayout {
+  int G = 0, nch = 0;
+  void* dmem = nullptr;
+  size_t dbytes = 0;
+  const int* boff = nullptr;
+  const uint4* blob = nullptr;
+};
+
+// True when every pattern of the set is one of the ring patterns (centre plus
+// 3 consecutive neighbours); ring_of[p] receives its ring index.
+bool tm_supports(const uint8_t* taps, int P, std::vector<int>& ring_of);
+pp_status tm_prepare();
+pp_status tm_build(TmLayout* T, const pp_packed* pk, const std::vector<int>& ring_of, cudaStream_t stream);
+pp_status tm_launch(const TmLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
+                    int H, int W, int flags, cudaStream_t stream);
 
 }  // namespace ppc

@@ -33,6 +33,10 @@ PP_ERR_UNSUPPORTED = 6
 PP_ERR_CUDA = 7
 PP_ERR_OOM = 8
 
+PP_KERNEL_AUTO = 0
+PP_KERNEL_TMEM = 1
+PP_KERNEL_REGISTER = 2
+
 PP_ADD_SKIP = 1
 PP_RELU = 2
 PP_POOL2 = 4
@@ -53,6 +57,8 @@ _SIGS = {
     "pp_layer_create": ([_P, _P, _P, _PP], _I),
     "pp_layer_info": ([_P, _P, _P, _P], _I),
     "pp_conv_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
+    "pp_layer_set_kernel": ([_P, _I], _I),
+    "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_destroy": ([_P], None),
     "pp_dense_create": ([_P, _P, _I, _I, _P, _PP], _I),
     "pp_dense_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
@@ -197,6 +203,16 @@ def pp_layer_info(layer):
 def pp_conv_forward(layer, x, y, skip, N, H, W, flags, stream=None):
     _check(lib.pp_conv_forward(layer, _dp(x), _dp(y), _dp(skip), N, H, W, flags, _stream(stream)),
            "pp_conv_forward")
+
+
+def pp_layer_set_kernel(layer, kernel: int):
+    _check(lib.pp_layer_set_kernel(layer, kernel), "pp_layer_set_kernel")
+
+
+def pp_layer_kernel(layer) -> int:
+    k = _I()
+    _check(lib.pp_layer_kernel(layer, ctypes.byref(k)), "pp_layer_kernel")
+    return k.value
 
 
 def pp_layer_destroy(layer):

@@ -35,9 +35,11 @@ def dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def run_layer(pp, runner, layer, x, skip=None, relu=False, pool=False):
+def run_layer(pp, runner, layer, x, skip=None, relu=False, pool=False, kernel=None):
     L = runner.DeviceLayer(layer)
     try:
+        if kernel is not None:
+            pp.pp_layer_set_kernel(L.handle, kernel)
         N, _, H, W = x.shape
         Ho, Wo = (H // 2, W // 2) if pool else (H, W)
         y = torch.full((N, layer.Co, Ho, Wo), float("nan"), device="cuda")
@@ -80,6 +82,41 @@ def test_layer_parity_small(pp, runner, oracle_mod, case, flags):
     check_within(g, y, s, f"{case} {flags}")
 
 
+@pytest.mark.parametrize("case", [c for c in SMALL if c[6]])
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+def test_register_kernel_on_ring_layers(pp, runner, oracle_mod, case, flags):
+    """Ring-set layers run the tensor-memory kernel by default; the register kernel must agree too."""
+    N, Ci, Co, H, W, P, ring, keep = case
+    if flags == "pool_relu" and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(sum(case[:5]) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=P, keep=keep, ring=ring)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=pp.PP_KERNEL_REGISTER)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
+    check_within(g, y, s, f"register kernel {case} {flags}")
+
+
+def test_kernel_selection(pp, runner):
+    rng = np.random.default_rng(2)
+    ring = runner.DeviceLayer(synth.small_random_layer(rng, 8, 8, ring=True))
+    other = runner.DeviceLayer(synth.small_random_layer(rng, 8, 8, P=8, ring=False))
+    try:
+        assert pp.pp_layer_kernel(ring.handle) == pp.PP_KERNEL_TMEM
+        assert pp.pp_layer_kernel(other.handle) == pp.PP_KERNEL_REGISTER
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_layer_set_kernel(other.handle, pp.PP_KERNEL_TMEM)
+        assert e.value.code == pp.PP_ERR_UNSUPPORTED
+        pp.pp_layer_set_kernel(ring.handle, pp.PP_KERNEL_REGISTER)
+        assert pp.pp_layer_kernel(ring.handle) == pp.PP_KERNEL_REGISTER
+        pp.pp_layer_set_kernel(ring.handle, pp.PP_KERNEL_AUTO)
+        assert pp.pp_layer_kernel(ring.handle) == pp.PP_KERNEL_TMEM
+    finally:
+        ring.close()
+        other.close()
+
+
 @pytest.mark.parametrize("ring", [True, False])
 def test_integer_layer_bit_exact(pp, runner, oracle_mod, ring):
     """Small-integer weights and inputs: every partial sum is exact in fp32, so GPU == oracle bit for bit."""
@@ -90,6 +127,9 @@ def test_integer_layer_bit_exact(pp, runner, oracle_mod, ring):
     g = run_layer(pp, runner, L, x)
     y, _ = oracle_layer_full(oracle_mod, L, x)
     assert (g.astype(np.float64) == y).all()
+    if ring:
+        g2 = run_layer(pp, runner, L, x, kernel=pp.PP_KERNEL_REGISTER)
+        assert (g2.astype(np.float64) == y).all()
 
 
 def test_all_pruned_layer_gives_bias(pp, runner, oracle_mod):
