@@ -248,9 +248,13 @@ def traffic_from_profile(kernel_hash: str):
 
 
 def kernel_source_hash():
+    """sha256 over the conv kernel sources (a profile taken on other sources is stale)."""
     import hashlib
-    with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", "conv.cu"), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()
+    h = hashlib.sha256()
+    for name in ("conv.cu", "conv_tm.cu", "internal.h"):
+        with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
 def bench_config(name, steps, warmup, flush, stream, hbm):
@@ -475,7 +479,7 @@ def main():
             "gpu_launches": len(spec.ops) * args.steps,
             "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
                          "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
-                         "kernel": "ppconv_kernel (pattern-pruned conv, all pruned ops of a step)",
+                         "kernel": "ppconv_tm_kernel / ppconv_kernel (pattern-pruned conv, all pruned ops of a step)",
                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
                          "hbm_peak_gbs": hbm, "hbm_peak_source": hbm_src},
             "layer_roofline_frac": layer_fracs,

@@ -377,11 +377,22 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_tm_kernel(const TmParams p
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase), "n"(TMEM_COLS));
 }
 
+// Number of CTAs sharing one output tile (split over input chunks), chosen by
+// a small cost model: resident waves (two CTAs per SM) x chunks per CTA, plus
+// about one chunk of work for the cluster reduction when split.
 int choose_split(int64_t base_ctas, int nch) {
-  const int sms = 152;
-  int ks = 1;
-  while (ks < MAX_SPLIT && ks * 2 <= nch && base_ctas * ks < 2 * sms) ks *= 2;
-  return ks;
+  const int64_t slots = 2 * 152;
+  int best = 1;
+  double best_t = 1e30;
+  for (int ks = 1; ks <= MAX_SPLIT && ks <= nch; ks *= 2) {
+    const double waves = (double)((base_ctas * ks + slots - 1) / slots);
+    const double t = waves * (double)((nch + ks - 1) / ks) + (ks > 1 ? 1.0 : 0.0);
+    if (t < best_t - 1e-9) {
+      best_t = t;
+      best = ks;
+    }
+  }
+  return best;
 }
 
 bool g_attr_done[64] = {};
