@@ -77,6 +77,7 @@ struct TmParams {
   int tiles_x;
   int flags;
   int ksplit, cpk;
+  int khalf;  // 1: maps at most 16 wide; the two warps of a group split each stage's channels
 };
 
 __host__ __device__ constexpr int ring_tap(int r, int s) {
@@ -218,14 +219,19 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_tm_kernel(const TmParams p
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int gq = warp & 3;   // group within the CTA = TMEM lane quadrant
-  const int sub = warp >> 2;  // which 16-column half of the tile
+  const int sub = warp >> 2;  // 16-column half of the tile, or (khalf) half of each stage's channels
   const int ly = lane & 15, lx = lane >> 4;
   const int ty = blockIdx.x / p.tiles_x, tx = blockIdx.x - ty * p.tiles_x;
-  const int r0 = ty * TILE_H, c0 = tx * TILE_W;
+  const int tile_w = p.khalf ? 16 : TILE_W;
+  const int r0 = ty * TILE_H, c0 = tx * tile_w;
+  const int cw = p.khalf ? 0 : sub * 16;  // this warp's column offset in the tile
   const int n = SPLIT ? blockIdx.z / p.ksplit : blockIdx.z;
   const int ks = SPLIT ? blockIdx.z - n * p.ksplit : 0;
   const int q = blockIdx.y * GROUPS + gq;
-  const bool active = q < p.G;
+  const bool grp = q < p.G;                          // the group exists
+  const bool compute = grp && c0 + cw < p.W;         // the warp's pixels overlap the image
+  const int chb = p.khalf ? sub * (CC / 2) : 0;      // channels of each stage this warp processes
+  const int che = p.khalf ? chb + CC / 2 : CC;
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -245,14 +251,14 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_tm_kernel(const TmParams p
     tm_wait_st();
   }
 
-  const int* boff = p.boff + (size_t)(active ? q : 0) * (p.nch + 1);
+  const int* boff = p.boff + (size_t)(grp ? q : 0) * (p.nch + 1);
   const int cbeg = ks * p.cpk;
   const int cend = min(p.nch, cbeg + p.cpk);
 
   auto issue = [&](int c) {
     unsigned char* st = smem + (c & 1) * STAGE_BYTES;
     stage_input(reinterpret_cast<float*>(st), p, n, c * CC, min(CC, p.Ci - c * CC), r0, c0);
-    if (active) {
+    if (grp) {
       // the two warps of a group split the blob copy
       const int b0 = __ldg(boff + c), b1 = __ldg(boff + c + 1);
       uint4* dst = reinterpret_cast<uint4*>(st + IN_BYTES + gq * BLOB_MAX);
@@ -270,19 +276,22 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_tm_kernel(const TmParams p
       cp_wait<0>();
     }
     __syncthreads();
-    if (active) {
+    if (compute) {
       const unsigned char* st = smem + (c & 1) * STAGE_BYTES;
-      const float* sin = reinterpret_cast<const float*>(st) + ly * SSTRIDE + sub * 16 + lx * PX;
+      const float* sin = reinterpret_cast<const float*>(st) + ly * SSTRIDE + cw + lx * PX;
       const unsigned char* blob = st + IN_BYTES + gq * BLOB_MAX;
       const unsigned char* bnd = blob;  // [CC][8]
       const int ntot = bnd[CC * 8 - 1];
       const unsigned char* slots = blob + 64;
       const float4* wts = reinterpret_cast<const float4*>(blob + 64 + ((ntot + 15) & ~15));
-      const int nvalid = min(CC, p.Ci - c * CC);
-      int e = 0;
-      for (int ch = 0; ch < nvalid; ++ch) {
+      const int nvalid = min(che, p.Ci - c * CC);
+      int e = chb > 0 ? bnd[(chb - 1) * 8 + 7] : 0;
+      for (int ch = chb; ch < nvalid; ++ch) {
         const unsigned char* bc = bnd + ch * 8;
         if (bc[7] == e) continue;  // no kept kernel of this group reads channel ch
+        // A slot updated in an earlier channel may be read again here: let its
+        // stores land first (within one channel every slot appears once).
+        tm_wait_st();
         const float* s = sin + ch * SCH;
         float2 E[3][5], O[3][4];
 #pragma unroll
@@ -312,12 +321,38 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_tm_kernel(const TmParams p
     }
     __syncthreads();
   }
+  // Every warp's accumulators are final once its stores have landed.
   tm_wait_st();
+  tm_fence_before();
+  __syncthreads();
+  tm_fence_after();
+  if (p.khalf) {
+    // The two warps of a group hold partial sums over different channels for
+    // the same pixels (same TMEM lanes): warp sub 0 adds its partner's columns.
+    if (grp && sub == 0) {
+      const uint32_t partner = tbase + ((uint32_t)(32 * gq) << 16) + (uint32_t)(F * PX);
+#pragma unroll 1
+      for (int j = 0; j < F; ++j) {
+        float a[PX], b[PX];
+        tm_ld8(wbase + j * PX, a);
+        tm_ld8(partner + j * PX, b);
+        tm_wait_ld();
+#pragma unroll
+        for (int k = 0; k < PX; ++k) a[k] += b[k];
+        tm_st8(wbase + j * PX, a);
+      }
+      tm_wait_st();
+    }
+    tm_fence_before();
+    __syncthreads();
+    tm_fence_after();
+  }
+  const bool fin = grp && (p.khalf ? sub == 0 : compute);  // warps that finalize outputs
 
   const int r = r0 + ly;
-  const int cb = c0 + sub * 16 + lx * PX;
+  const int cb = c0 + cw + lx * PX;
   if constexpr (!SPLIT) {
-    if (active) {
+    if (fin) {
 #pragma unroll 1
       for (int j = 0; j < F; ++j) {
         const int jr = q * F + j;
@@ -347,7 +382,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) ppconv_tm_kernel(const TmParams p
         for (int k = 0; k < PX; ++k) red[((warp * 8 + jj) * PX + k) * 32 + lane] = v[k];
       }
       cluster.sync();
-      if (active) {
+      if (fin) {
 #pragma unroll 1
         for (int jj = 0; jj < 8; ++jj) {
           const int j = half * 8 + jj;
@@ -504,9 +539,12 @@ pp_status tm_build(TmLayout* T, const pp_packed* pk, const std::vector<int>& rin
 
 pp_status tm_launch(const TmLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N, int H,
                     int W, int flags, cudaStream_t stream) {
-  const int tiles_y = (H + TILE_H - 1) / TILE_H, tiles_x = (W + TILE_W - 1) / TILE_W;
+  const int khalf = W <= 16 ? 1 : 0;
+  const int tile_w = khalf ? 16 : TILE_W;
+  const int tiles_y = (H + TILE_H - 1) / TILE_H, tiles_x = (W + tile_w - 1) / tile_w;
   if ((int64_t)tiles_y * tiles_x > INT32_MAX) return PP_ERR_UNSUPPORTED;
   TmParams p;
+  p.khalf = khalf;
   p.x = x;
   p.y = y;
   p.skip = (flags & PP_ADD_SKIP) ? skip : nullptr;

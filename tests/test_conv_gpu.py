@@ -62,6 +62,10 @@ SMALL = [
     (1, 35, 18, 33, 18, 8, True, 1.0),
     (3, 5, 7, 2, 3, 8, False, 0.9),
     (1, 64, 64, 12, 44, 8, True, 0.2),
+    (1, 40, 24, 14, 14, 8, True, 0.3),   # maps <= 16 wide: warps split each stage's channels
+    (2, 64, 64, 10, 16, 8, True, 0.5),
+    (1, 24, 20, 9, 17, 8, True, 0.6),    # 17 wide: the second tile half holds one column
+    (1, 3, 70, 6, 4, 8, True, 1.0),
 ]
 
 
