@@ -144,17 +144,28 @@ pp_status pp_layer_info(const pp_layer* layer, int* Co, int* Ci, int64_t* device
 pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H, int W,
                           int flags, void* stream);
 
-/* Which kernel pp_conv_forward runs for a layer.  PP_KERNEL_AUTO picks the
- * tensor-memory kernel when every pattern is a ring pattern (the centre tap
- * plus 3 consecutive of its 8 neighbours) and the register kernel otherwise.
- * Setting PP_KERNEL_TMEM on a layer whose patterns are not all ring patterns
- * returns PP_ERR_UNSUPPORTED.  Both kernels compute the same convolution. */
+/* Which kernel pp_conv_forward runs for a layer.  All compute the same
+ * convolution within the documented fp32 bound.
+ *   PP_KERNEL_TC        implicit GEMM on the tensor cores over the 9 taps
+ *                       (zeros where pruned), 3xTF32 for fp32 accuracy; any
+ *                       pattern set; needs Ci >= 8.
+ *   PP_KERNEL_TMEM      FP32 FMA over kept taps only, accumulators in tensor
+ *                       memory; ring patterns only (the centre tap plus 3
+ *                       consecutive of its 8 neighbours).
+ *   PP_KERNEL_REGISTER  FP32 FMA over kept taps, accumulators in registers;
+ *                       any pattern set.
+ * PP_KERNEL_AUTO picks by an estimate of each kernel's time for the layer's
+ * density.  Setting a kernel the layer cannot run returns PP_ERR_UNSUPPORTED. */
 #define PP_KERNEL_AUTO 0
 #define PP_KERNEL_TMEM 1
 #define PP_KERNEL_REGISTER 2
+#define PP_KERNEL_TC 3
 pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
-/* The kernel that pp_conv_forward will run (PP_KERNEL_TMEM or PP_KERNEL_REGISTER). */
+/* The kernel that pp_conv_forward will run (PP_KERNEL_TC, _TMEM or _REGISTER). */
 pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
+/* Synchronous: *device_error = 0 unless a kernel of this layer gave up a
+ * bounded wait (its output is then invalid); the word is cleared by the read. */
+pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);
 
 void pp_layer_destroy(pp_layer* layer);
 

@@ -395,8 +395,11 @@ struct pp_layer {
   int Co = 0, Ci = 0;
   int mode = MODE_GENERIC;
   bool tm_ok = false;    // ring-set layer: the tensor-memory kernel can run it
-  bool use_tm = false;
+  bool tc_ok = false;    // the tensor-core kernel can run it
+  int kernel = 2;        // PP_KERNEL_TMEM / _REGISTER / _TC
+  int auto_kernel = 2;
   ppc::TmLayout tm;
+  ppc::TcLayout tc;
   int G = 0, nch = 0;
   int cc = CC;  // input channels per stage
   int64_t nE = 0;
@@ -550,13 +553,14 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   if ((flags & PP_ADD_SKIP) && !skip) return PP_ERR_INVALID_ARG;
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   if (((uintptr_t)y & 15) || ((uintptr_t)x & 3)) return PP_ERR_INVALID_ARG;
-  if (L->use_tm) {
+  if (L->kernel == PP_KERNEL_TMEM || L->kernel == PP_KERNEL_TC) {
     ppc::LayerMeta M;
     M.Co = L->Co;
     M.Ci = L->Ci;
     M.perm = L->perm;
     M.bias = L->has_bias ? L->bias : nullptr;
-    return ppc::tm_launch(L->tm, M, x, y, skip, N, H, W, flags, stream);
+    return L->kernel == PP_KERNEL_TC ? ppc::tc_launch(L->tc, M, x, y, skip, N, H, W, flags, stream)
+                                     : ppc::tm_launch(L->tm, M, x, y, skip, N, H, W, flags, stream);
   }
   const int tiles_y = (H + TH - 1) / TH, tiles_x = (W + TW - 1) / TW;
   if ((int64_t)tiles_y * tiles_x > INT32_MAX) return PP_ERR_UNSUPPORTED;
@@ -650,41 +654,66 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
     st = ppc::tm_prepare();
     if (st == PP_OK) st = ppc::tm_build(&L->tm, pk, rmap, (cudaStream_t)stream);
     L->tm_ok = st == PP_OK;
-    L->use_tm = L->tm_ok;
+  }
+  if (st == PP_OK && pk->Ci >= 8) {
+    st = ppc::tc_prepare();
+    if (st == PP_OK) st = ppc::tc_build(&L->tc, pk, (cudaStream_t)stream);
+    L->tc_ok = st == PP_OK;
   }
   if (st != PP_OK) {
     pp_layer_destroy(L);
     return st;
   }
+  // Kernel choice by estimated SM cycles per pixel: the tensor cores run the
+  // dense 9-tap contraction (filters padded to 128, channels to 8) three times
+  // at ~1800 multiply-adds per cycle; the FMA kernels run only the kept taps
+  // at a quarter of the 128 FMA lanes (what they reach on these layers).
+  const double nk = (double)pk->kidx.size();
+  const double tc_cycles = 27.0 * (double)((pk->Co + 127) / 128 * 128) * (double)((pk->Ci + 7) / 8 * 8) / 1800.0;
+  const double fma_cycles = 4.0 * nk / 32.0;
+  L->auto_kernel = (L->tc_ok && tc_cycles < fma_cycles) ? PP_KERNEL_TC : (L->tm_ok ? PP_KERNEL_TMEM : PP_KERNEL_REGISTER);
+  L->kernel = L->auto_kernel;
   *out = L;
   return PP_OK;
 }
 
 extern "C" pp_status pp_layer_set_kernel(pp_layer* L, int kernel) {
   if (!L) return PP_ERR_INVALID_ARG;
-  if (kernel == PP_KERNEL_AUTO || kernel == PP_KERNEL_TMEM) {
-    if (kernel == PP_KERNEL_TMEM && !L->tm_ok) return PP_ERR_UNSUPPORTED;
-    L->use_tm = L->tm_ok;
-    return PP_OK;
+  switch (kernel) {
+    case PP_KERNEL_AUTO: L->kernel = L->auto_kernel; return PP_OK;
+    case PP_KERNEL_TMEM:
+      if (!L->tm_ok) return PP_ERR_UNSUPPORTED;
+      L->kernel = kernel;
+      return PP_OK;
+    case PP_KERNEL_TC:
+      if (!L->tc_ok) return PP_ERR_UNSUPPORTED;
+      L->kernel = kernel;
+      return PP_OK;
+    case PP_KERNEL_REGISTER: L->kernel = kernel; return PP_OK;
+    default: return PP_ERR_INVALID_ARG;
   }
-  if (kernel == PP_KERNEL_REGISTER) {
-    L->use_tm = false;
-    return PP_OK;
-  }
-  return PP_ERR_INVALID_ARG;
 }
 
 extern "C" pp_status pp_layer_kernel(const pp_layer* L, int* kernel) {
   if (!L || !kernel) return PP_ERR_INVALID_ARG;
-  *kernel = L->use_tm ? PP_KERNEL_TMEM : PP_KERNEL_REGISTER;
+  *kernel = L->kernel;
   return PP_OK;
+}
+
+extern "C" pp_status pp_layer_device_status(const pp_layer* L, int* device_error) {
+  if (!L || !device_error) return PP_ERR_INVALID_ARG;
+  *device_error = 0;
+  if (!L->tc_ok) return PP_OK;
+  pp_status st = ppc::tc_status(L->tc, device_error);
+  if (st == PP_OK && *device_error && cudaMemset(L->tc.status, 0, sizeof(int)) != cudaSuccess) return PP_ERR_CUDA;
+  return st;
 }
 
 extern "C" pp_status pp_layer_info(const pp_layer* L, int* Co, int* Ci, int64_t* device_bytes) {
   if (!L) return PP_ERR_INVALID_ARG;
   if (Co) *Co = L->Co;
   if (Ci) *Ci = L->Ci;
-  if (device_bytes) *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes);
+  if (device_bytes) *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes + L->tc.dbytes);
   return PP_OK;
 }
 
@@ -697,6 +726,7 @@ extern "C" void pp_layer_destroy(pp_layer* L) {
   if (!L) return;
   if (L->dmem) cudaFree(L->dmem);
   if (L->tm.dmem) cudaFree(L->tm.dmem);
+  if (L->tc.dmem) cudaFree(L->tc.dmem);
   delete L;
 }
 

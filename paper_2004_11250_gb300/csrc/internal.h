@@ -47,6 +47,21 @@ struct TmLayout {
   const uint4* blob = nullptr;
 };
 
+// Dense per-tap tf32 hi/lo weight tiles of the tensor-core kernel (conv_tc.cu).
+struct TcLayout {
+  int MT = 0, nch = 0;
+  void* dmem = nullptr;
+  size_t dbytes = 0;
+  const unsigned char* a = nullptr;
+  int* status = nullptr;  // device word, nonzero after a timed-out wait
+};
+
+pp_status tc_prepare();
+pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream);
+pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
+                    int H, int W, int flags, cudaStream_t stream);
+pp_status tc_status(const TcLayout& T, int* device_error);
+
 // True when every pattern of the set is one of the ring patterns (centre plus
 // 3 consecutive neighbours); ring_of[p] receives its ring index.
 bool tm_supports(const uint8_t* taps, int P, std::vector<int>& ring_of);

@@ -36,6 +36,7 @@ PP_ERR_OOM = 8
 PP_KERNEL_AUTO = 0
 PP_KERNEL_TMEM = 1
 PP_KERNEL_REGISTER = 2
+PP_KERNEL_TC = 3
 
 PP_ADD_SKIP = 1
 PP_RELU = 2
@@ -59,6 +60,7 @@ _SIGS = {
     "pp_conv_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
     "pp_layer_set_kernel": ([_P, _I], _I),
     "pp_layer_kernel": ([_P, _P], _I),
+    "pp_layer_device_status": ([_P, _P], _I),
     "pp_layer_destroy": ([_P], None),
     "pp_dense_create": ([_P, _P, _I, _I, _P, _PP], _I),
     "pp_dense_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
@@ -213,6 +215,12 @@ def pp_layer_kernel(layer) -> int:
     k = _I()
     _check(lib.pp_layer_kernel(layer, ctypes.byref(k)), "pp_layer_kernel")
     return k.value
+
+
+def pp_layer_device_status(layer) -> int:
+    v = _I()
+    _check(lib.pp_layer_device_status(layer, ctypes.byref(v)), "pp_layer_device_status")
+    return v.value
 
 
 def pp_layer_destroy(layer):

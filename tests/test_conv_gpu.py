@@ -102,6 +102,34 @@ def test_register_kernel_on_ring_layers(pp, runner, oracle_mod, case, flags):
     check_within(g, y, s, f"register kernel {case} {flags}")
 
 
+@pytest.mark.parametrize("case", [c for c in SMALL if c[1] >= 8])
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+def test_tensor_core_kernel(pp, runner, oracle_mod, case, flags):
+    """The 3xTF32 implicit-GEMM kernel on every small case with at least 8 input channels."""
+    N, Ci, Co, H, W, P, ring, keep = case
+    if flags == "pool_relu" and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(7 * sum(case[:5]) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=P, keep=keep, ring=ring)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=pp.PP_KERNEL_TC)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
+    check_within(g, y, s, f"tensor-core kernel {case} {flags}")
+
+
+def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
+    """Shapes that exercise every tile width (16/32/64/128 pixels) and the cluster split of the channel chunks."""
+    rng = np.random.default_rng(31)
+    for (N, Ci, Co, H, W) in ((1, 72, 130, 12, 14), (1, 40, 64, 20, 30), (1, 24, 128, 9, 60), (1, 16, 33, 5, 140),
+                              (2, 136, 200, 7, 9)):
+        L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.4)
+        x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+        g = run_layer(pp, runner, L, x, None, True, False, kernel=pp.PP_KERNEL_TC)
+        y, s = oracle_layer_full(oracle_mod, L, x, None, True, False)
+        check_within(g, y, s, f"tensor-core kernel {(N, Ci, Co, H, W)}")
+
+
 def test_kernel_selection(pp, runner):
     rng = np.random.default_rng(2)
     ring = runner.DeviceLayer(synth.small_random_layer(rng, 8, 8, ring=True))
@@ -116,6 +144,9 @@ def test_kernel_selection(pp, runner):
         assert pp.pp_layer_kernel(ring.handle) == pp.PP_KERNEL_REGISTER
         pp.pp_layer_set_kernel(ring.handle, pp.PP_KERNEL_AUTO)
         assert pp.pp_layer_kernel(ring.handle) == pp.PP_KERNEL_TMEM
+        pp.pp_layer_set_kernel(ring.handle, pp.PP_KERNEL_TC)
+        assert pp.pp_layer_kernel(ring.handle) == pp.PP_KERNEL_TC
+        assert pp.pp_layer_device_status(ring.handle) == 0
     finally:
         ring.close()
         other.close()
@@ -134,6 +165,9 @@ def test_integer_layer_bit_exact(pp, runner, oracle_mod, ring):
     if ring:
         g2 = run_layer(pp, runner, L, x, kernel=pp.PP_KERNEL_REGISTER)
         assert (g2.astype(np.float64) == y).all()
+    # integers below 2^11 are exact in tf32, so the 3xTF32 kernel is exact too
+    g3 = run_layer(pp, runner, L, x, kernel=pp.PP_KERNEL_TC)
+    assert (g3.astype(np.float64) == y).all()
 
 
 def test_all_pruned_layer_gives_bias(pp, runner, oracle_mod):
