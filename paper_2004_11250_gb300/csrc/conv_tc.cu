@@ -49,34 +49,38 @@
 
 namespace {
 
-constexpr int TC_M = 128;          // filters per CTA (MMA M)
 constexpr int KC = 8;              // input channels per chunk (MMA K for tf32)
 constexpr int NTAP = 9;
-constexpr int NCOL = 256;          // TMEM columns = accumulator pixels per CTA
-constexpr int NTHREADS = 128;
-constexpr int A_TILE = TC_M * KC * 4;             // one tap, one of hi/lo: 4 KB
-constexpr int A_BYTES = NTAP * 2 * A_TILE;        // 72 KB per chunk
-constexpr int MAX_SPLIT = 8;
-constexpr long WAIT_LIMIT = 1L << 24;             // mbarrier polls before giving up
+constexpr int NCOL = 256;          // TMEM columns of one accumulator buffer
+constexpr int NLOAD = 128;         // loader threads (warps 0-3)
+constexpr int MMA_WARP = 4;        // warp 4: TMEM owner and MMA issuer
+constexpr int NTHREADS = 288;      // + epilogue warps 5-8
+constexpr long WAIT_LIMIT = 1L << 22;  // mbarrier polls before a wait gives up
+
+// Orientation of the GEMM on the tensor core.
+//   ORI_FP: M = 128 filters, N = TW pixels of one output row (narrow maps)
+//   ORI_PF: M = 128 pixels of one output row, N = FB filters (wide maps)
+enum { ORI_FP = 0, ORI_PF = 1 };
 
 struct TcParams {
   const float* x;
   float* y;
   const float* skip;
-  const unsigned char* a;  // [MT][nch][9][2][128 x 8] canonical tiles
-  const int* perm;         // [Co]
-  const float* bias;       // [Co] reordered, or null
-  int* status;             // device status word (nonzero after a timed-out wait)
+  const unsigned char* wt;  // [nfb][nch][9][2][FB x 8] canonical tiles
+  const int* perm;          // [Co]
+  const float* bias;        // [Co] reordered, or null
+  int* status;              // device status word (nonzero after a timed-out wait)
   int N, Ci, Co, H, W;
-  int nch, MT;
-  int tiles_x, tiles_y;
+  int nch, nfb, FB;
+  int tiles_x, tiles_y, ntiles;
   int flags;
-  int ksplit, cpk;
 };
 
+__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
 // Shared-memory matrix descriptor, K-major, no swizzle: core matrices of 8 rows
-// x 16 bytes; lbo = byte distance between the two K halves, sbo = between
-// groups of 8 rows.
+// x 16 bytes; lbo = byte distance between the two K halves, sbo = 128 between
+// groups of 8 rows; bit 46 = descriptor version of this architecture.
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo) {
   uint64_t d = (uint64_t)((addr >> 4) & 0x3FFF);
   d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
@@ -90,8 +94,6 @@ __host__ __device__ constexpr uint32_t idesc_tf32(int m, int n) {
   return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
-__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
 __device__ __forceinline__ void mbar_init(uint32_t a, int count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count));
 }
@@ -103,22 +105,13 @@ __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
                : "memory");
   return ok != 0;
 }
-// Bounded wait; returns false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
-  for (long i = 0; i < WAIT_LIMIT; ++i)
-    if (mbar_try(a, parity)) return true;
-  return false;
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
 }
-
-__device__ __forceinline__ void cp4(void* s, const void* g, bool valid) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(su32(s)), "l"(g), "r"(valid ? 4 : 0));
-}
-__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-__device__ __forceinline__ void cp_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
 
 __device__ __forceinline__ void tm_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tm_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
+__device__ __forceinline__ void tm_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tm_ld16(uint32_t ta, float (&v)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -126,332 +119,319 @@ __device__ __forceinline__ void tm_ld16(uint32_t ta, float (&v)[16]) {
         "=f"(v[9]), "=f"(v[10]), "=f"(v[11]), "=f"(v[12]), "=f"(v[13]), "=f"(v[14]), "=f"(v[15])
       : "r"(ta));
 }
-__device__ __forceinline__ void tm_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-
 __device__ __forceinline__ void mma_tf32(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc) {
   asm volatile(
       "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p; }" ::"r"(d),
       "l"(a), "l"(b), "r"(id), "r"(acc));
 }
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
 
-template <int TW>
+// Geometry of one instantiation.  TW pixels per output row segment, FB filters
+// per block, R row segments per tile (one accumulator column range each).
+template <int ORI, int TW, int FB>
 struct Geo {
-  static constexpr int R = NCOL / TW;          // output rows per CTA
-  static constexpr int BROWS = R + 2;
-  static constexpr int BCOLS = TW + 2;
-  static constexpr int NPIX = BROWS * BCOLS;   // pixels of the staged input tile
-  static constexpr int B_HALF = NPIX * 16;     // bytes of one K half (4 channels) of one of hi / lo
-  static constexpr int B_BYTES = 2 * B_HALF;   // hi or lo tile (8 channels)
-  static constexpr int STAGE = A_BYTES + 2 * B_BYTES;
-  static constexpr int SMEM = 2 * STAGE;
-  static constexpr int RED = TC_M * NCOL * 4;  // split-K partial sums of the CTA
-  static constexpr int SMEM_ALLOC = (SMEM > RED ? SMEM : RED) + 1024;
+  static_assert(ORI == ORI_FP ? FB == 128 : TW == 128, "orientation needs a 128-row M side");
+  static constexpr int SEGC = ORI == ORI_FP ? TW : FB;   // accumulator columns per row segment
+  static constexpr int R = NCOL / SEGC;                   // row segments per tile
+  static constexpr int BROWS = R + 2, BCOLS = TW + 2;
+  static constexpr int NPIX = BROWS * BCOLS;              // staged input pixels
+  static constexpr int IN_HALF = NPIX * 16;               // one K half (4 channels) of hi or lo
+  static constexpr int IN_BYTES = 2 * IN_HALF;            // hi or lo, 8 channels
+  static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo
+  static constexpr int W_BYTES = NTAP * 2 * W_TILE;       // weights of one chunk
+  static constexpr int STAGE = W_BYTES + 2 * IN_BYTES;
+  static constexpr int SMEM_ALLOC = 2 * STAGE + 1024;
+  static constexpr uint32_t IDESC = ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB);
 };
 
-// Epilogue of 16 consecutive pixels (one row, columns c .. c+15 of the tile) of one filter.
-__device__ __forceinline__ void store16(const TcParams& p, int n, int m_global, float (&v)[16], int row, int col) {
-  if (m_global >= p.Co || row >= p.H) return;
-  const int o = __ldg(p.perm + m_global);
-  const float b = p.bias ? __ldg(p.bias + m_global) : 0.f;
-#pragma unroll
-  for (int k = 0; k < 16; ++k) v[k] += b;
-  if (p.flags & PP_ADD_SKIP) {
-    const float* sk = p.skip + (((size_t)n * p.Co + o) * p.H + row) * p.W;
-#pragma unroll
-    for (int k = 0; k < 16; ++k)
-      if (col + k < p.W) v[k] += __ldg(sk + col + k);
-  }
-  if (p.flags & PP_RELU) {
-#pragma unroll
-    for (int k = 0; k < 16; ++k) v[k] = fmaxf(v[k], 0.f);
-  }
-  float* yo = p.y + (((size_t)n * p.Co + o) * p.H + row) * p.W;
-  if (col + 16 <= p.W && (p.W & 3) == 0 && (col & 3) == 0) {
-#pragma unroll
-    for (int k = 0; k < 16; k += 4) *reinterpret_cast<float4*>(yo + col + k) = make_float4(v[k], v[k + 1], v[k + 2], v[k + 3]);
-  } else {
-#pragma unroll
-    for (int k = 0; k < 16; ++k)
-      if (col + k < p.W) yo[col + k] = v[k];
-  }
+struct Tile {
+  int n, r0, c0, fb;
+};
+__device__ __forceinline__ Tile tile_of(const TcParams& p, int t, int R, int TW) {
+  Tile T;
+  T.fb = t % p.nfb;
+  t /= p.nfb;
+  const int tx = t % p.tiles_x;
+  t /= p.tiles_x;
+  const int ty = t % p.tiles_y;
+  T.n = t / p.tiles_y;
+  T.r0 = ty * R;
+  T.c0 = tx * TW;
+  return T;
 }
 
-// Pooled epilogue: rows row, row+1 (a, b), columns col .. col+15 -> 8 outputs.
-__device__ __forceinline__ void store16_pool(const TcParams& p, int n, int m_global, float (&a)[16], float (&b)[16],
-                                             int row, int col) {
-  if (m_global >= p.Co || row >= p.H) return;
-  const int o = __ldg(p.perm + m_global);
-  const float bs = p.bias ? __ldg(p.bias + m_global) : 0.f;
-#pragma unroll
-  for (int k = 0; k < 16; ++k) {
-    a[k] += bs;
-    b[k] += bs;
-  }
-  if (p.flags & PP_ADD_SKIP) {
-    const float* s0 = p.skip + (((size_t)n * p.Co + o) * p.H + row) * p.W;
-    const float* s1 = s0 + p.W;
-#pragma unroll
-    for (int k = 0; k < 16; ++k)
-      if (col + k < p.W) {
-        a[k] += __ldg(s0 + col + k);
-        b[k] += __ldg(s1 + col + k);
-      }
-  }
-  if (p.flags & PP_RELU) {
-#pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      a[k] = fmaxf(a[k], 0.f);
-      b[k] = fmaxf(b[k], 0.f);
-    }
-  }
-  const int Ho = p.H / 2, Wo = p.W / 2;
-  float* yo = p.y + (((size_t)n * p.Co + o) * Ho + (row >> 1)) * Wo;
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const int pc = (col >> 1) + k;
-    if (pc < Wo) yo[pc] = fmaxf(fmaxf(a[2 * k], a[2 * k + 1]), fmaxf(b[2 * k], b[2 * k + 1]));
-  }
-}
-
-template <int TW, bool SPLIT>
+template <int ORI, int TW, int FB>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p) {
-  using G = Geo<TW>;
+  using G = Geo<ORI, TW, FB>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar_a[2];    // weights of a stage have arrived
-  __shared__ __align__(8) uint64_t bar_mma[2];  // MMAs reading a stage are done
+  __shared__ __align__(8) uint64_t full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
   __shared__ uint32_t tmem_s;
-  __shared__ int abort_s;
+  __shared__ volatile int abort_s;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int tile = blockIdx.x;
-  const int ty = tile / p.tiles_x, tx = tile - ty * p.tiles_x;
-  const int r0 = ty * G::R, c0 = tx * TW;
-  const int mt = blockIdx.y;
-  const int n = SPLIT ? blockIdx.z / p.ksplit : blockIdx.z;
-  const int ks = SPLIT ? blockIdx.z - n * p.ksplit : 0;
-  const int cbeg = ks * p.cpk;
-  const int cend = min(p.nch, cbeg + p.cpk);
+
+  // Bounded wait that gives up early once another role has aborted.
+  auto wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+    const uint32_t a = su32(bar);
+    for (long i = 0; i < WAIT_LIMIT; ++i) {
+      if (mbar_try(a, parity)) return true;
+      if ((i & 255) == 255 && abort_s) return false;
+    }
+    abort_s = 1;
+    atomicExch(p.status, 1);
+    return false;
+  };
 
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
-      mbar_init(su32(&bar_a[s]), 1);
-      mbar_init(su32(&bar_mma[s]), 1);
+      mbar_init(su32(&full[s]), NLOAD);
+      mbar_init(su32(&empty[s]), 1);
+      mbar_init(su32(&acc_full[s]), 1);
+      mbar_init(su32(&acc_empty[s]), 128);
     }
+    mbar_init(su32(&done_bar), 1);
     abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 0) {
+  if (warp == MMA_WARP) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&tmem_s)),
-                 "n"(NCOL));
+                 "n"(2 * NCOL));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   tm_fence_before();
   __syncthreads();
   tm_fence_after();
   const uint32_t tmem = tmem_s;
+  const int nmine = p.ntiles > (int)blockIdx.x ? (p.ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
-  // Stage s of chunk c: weights by one bulk copy, input tile by cp.async.
-  auto load = [&](int c, int s) {
-    unsigned char* st = smem + s * G::STAGE;
-    if (tid == 0) {
-      const unsigned char* src = p.a + ((size_t)mt * p.nch + c) * A_BYTES;
-      const uint32_t bar = su32(&bar_a[s]);
-      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(A_BYTES) : "memory");
-      asm volatile(
-          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(su32(st)),
-          "l"(src), "r"(A_BYTES), "r"(bar)
-          : "memory");
-    }
-    float* bh = reinterpret_cast<float*>(st + A_BYTES);
-    const int i0 = c * KC;
-    const float* xb = p.x + (size_t)n * p.Ci * p.H * p.W;
-    const int total = KC * G::NPIX;
-    for (int e = tid; e < total; e += NTHREADS) {
-      const int k = e / G::NPIX;
-      const int pix = e - k * G::NPIX;
-      const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
-      const int r = r0 - 1 + br, cc = c0 - 1 + bc, ch = i0 + k;
-      const bool ok = ch < p.Ci && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
-      cp4(bh + (k >> 2) * (G::NPIX * 4) + pix * 4 + (k & 3), ok ? xb + ((size_t)ch * p.H + r) * p.W + cc : p.x, ok);
-    }
-    cp_commit();
-  };
-
-  bool ok = true;
-  if (cbeg < cend) load(cbeg, 0);
-  for (int c = cbeg; c < cend; ++c) {
-    const int s = (c - cbeg) & 1;
-    const int use = (c - cbeg) >> 1;  // how many times stage s was used before
-    unsigned char* st = smem + s * G::STAGE;
-    cp_wait_all();
-    __syncthreads();
-    // split the input tile into hi (in place) and lo
-    {
-      float4* bh = reinterpret_cast<float4*>(st + A_BYTES);
-      float4* bl = reinterpret_cast<float4*>(st + A_BYTES + G::B_BYTES);
-      for (int e = tid; e < 2 * G::NPIX; e += NTHREADS) {
-        const float4 v = bh[e];
-        float4 h;
-        h.x = __uint_as_float(__float_as_uint(v.x) & 0xFFFFE000u);
-        h.y = __uint_as_float(__float_as_uint(v.y) & 0xFFFFE000u);
-        h.z = __uint_as_float(__float_as_uint(v.z) & 0xFFFFE000u);
-        h.w = __uint_as_float(__float_as_uint(v.w) & 0xFFFFE000u);
-        bh[e] = h;
-        bl[e] = make_float4(v.x - h.x, v.y - h.y, v.z - h.z, v.w - h.w);
-      }
-    }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    __syncthreads();
-    if (tid == 0) {
-      if (!mbar_wait(su32(&bar_a[s]), (uint32_t)(use & 1))) abort_s = 1;
-      if (!abort_s) {
-        tm_fence_after();
-        const uint32_t abase = su32(st);
-        const uint32_t bhi = su32(st + A_BYTES), blo = su32(st + A_BYTES + G::B_BYTES);
-        constexpr uint32_t id = idesc_tf32(TC_M, TW);
-#pragma unroll 1
-        for (int t = 0; t < NTAP; ++t) {
-          const int dy = t / 3, dx = t % 3;
-          const uint64_t ahi = smem_desc(abase + (t * 2 + 0) * A_TILE, TC_M * 16);
-          const uint64_t alo = smem_desc(abase + (t * 2 + 1) * A_TILE, TC_M * 16);
-#pragma unroll 1
-          for (int rr = 0; rr < G::R; ++rr) {
-            const uint32_t off = (uint32_t)(((rr + dy) * G::BCOLS + dx) * 16);
-            const uint64_t bdh = smem_desc(bhi + off, G::B_HALF);
-            const uint64_t bdl = smem_desc(blo + off, G::B_HALF);
-            const uint32_t d = tmem + (uint32_t)(rr * TW);
-            const uint32_t first = (c == cbeg && t == 0) ? 0u : 1u;
-            mma_tf32(d, ahi, bdh, id, first);
-            mma_tf32(d, alo, bdh, id, 1u);
-            mma_tf32(d, ahi, bdl, id, 1u);
-          }
+  if (warp < 4) {
+    // ------------------------------------------------------------ loaders
+    int g = 0;  // chunk sequence number of this CTA
+    for (int i = 0; i < nmine && !abort_s; ++i) {
+      const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
+      const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
+      for (int c = 0; c < p.nch; ++c, ++g) {
+        const int s = g & 1, use = g >> 1;
+        if (use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1))) break;
+        unsigned char* st = smem + s * G::STAGE;
+        if (tid == 0) {
+          const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * G::W_BYTES;
+          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(&full[s])),
+                       "r"(G::W_BYTES)
+                       : "memory");
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                  su32(st)),
+              "l"(src), "r"(G::W_BYTES), "r"(su32(&full[s]))
+              : "memory");
         }
-        asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                         su32(&bar_mma[s]))
-                     : "memory");
-      }
-    }
-    __syncthreads();
-    if (abort_s) {
-      ok = false;
-      break;
-    }
-    // Load the chunk after this one into the other stage once the MMAs that
-    // read it (chunk c - 1) are done.
-    if (c + 1 < cend) {
-      const int s2 = s ^ 1;
-      if (c > cbeg) {
-        const int use2 = (c - 1 - cbeg) >> 1;
-        if (!mbar_wait(su32(&bar_mma[s2]), (uint32_t)(use2 & 1))) {
-          if (tid == 0) abort_s = 1;
+        // input tile: item = (K half, pixel); 4 channels of one pixel, split into hi / lo
+        float4* hi = reinterpret_cast<float4*>(st + G::W_BYTES);
+        float4* lo = reinterpret_cast<float4*>(st + G::W_BYTES + G::IN_BYTES);
+        const int ch0 = c * KC;
+        for (int it = tid; it < 2 * G::NPIX; it += NLOAD) {
+          const int kh = it >= G::NPIX ? 1 : 0;
+          const int pix = it - kh * G::NPIX;
+          const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
+          const int r = T.r0 - 1 + br, cc = T.c0 - 1 + bc;
+          float v[4];
+          const bool inside = (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int ch = ch0 + kh * 4 + k;
+            v[k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
+          }
+          float4 h, l;
+          h.x = __uint_as_float(__float_as_uint(v[0]) & 0xFFFFE000u);
+          h.y = __uint_as_float(__float_as_uint(v[1]) & 0xFFFFE000u);
+          h.z = __uint_as_float(__float_as_uint(v[2]) & 0xFFFFE000u);
+          h.w = __uint_as_float(__float_as_uint(v[3]) & 0xFFFFE000u);
+          l = make_float4(v[0] - h.x, v[1] - h.y, v[2] - h.z, v[3] - h.w);
+          hi[it] = h;
+          lo[it] = l;
         }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        if (tid == 0)
+          ;  // thread 0 arrived with the transaction count above
+        else
+          mbar_arrive(su32(&full[s]));
+      }
+    }
+  } else if (warp == MMA_WARP) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int g = 0;
+      for (int i = 0; i < nmine && !abort_s; ++i) {
+        const int b = i & 1, ub = i >> 1;
+        if (ub > 0 && !wait(&acc_empty[b], (uint32_t)((ub - 1) & 1))) break;
         tm_fence_after();
-      }
-      __syncthreads();
-      if (abort_s) {
-        ok = false;
-        break;
-      }
-      load(c + 1, s2);
-    }
-  }
-  // Wait for the last chunk's MMAs (they complete after all earlier ones).
-  if (ok && cend > cbeg) {
-    const int last = cend - 1 - cbeg;
-    if (!mbar_wait(su32(&bar_mma[last & 1]), (uint32_t)((last >> 1) & 1))) ok = false;
-    tm_fence_after();
-  }
-  if (!ok && tid == 0) atomicExch(p.status, 1);
-  cp_wait_all();
-  __syncthreads();
-
-  // Epilogue: thread = filter (TMEM lane 32 * warp + lane); pixels along columns.
-  const int m = warp * 32 + lane;
-  const int mg = mt * TC_M + m;
-  const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
-  const bool pool = p.flags & PP_POOL2;
-  if constexpr (!SPLIT) {
-    if (ok) {
-      if (!pool) {
-#pragma unroll 1
-        for (int rr = 0; rr < G::R; ++rr)
-#pragma unroll 1
-          for (int cc = 0; cc < TW; cc += 16) {
-            float v[16];
-            tm_ld16(lane_addr + (uint32_t)(rr * TW + cc), v);
-            tm_wait_ld();
-            store16(p, n, mg, v, r0 + rr, c0 + cc);
+        const uint32_t dbase = tmem + (uint32_t)(b * NCOL);
+        bool okc = true;
+        for (int c = 0; c < p.nch; ++c, ++g) {
+          const int s = g & 1, use = g >> 1;
+          if (!wait(&full[s], (uint32_t)(use & 1))) {
+            okc = false;
+            break;
           }
-      } else {
+          tm_fence_after();
+          const unsigned char* st = smem + s * G::STAGE;
+          const uint32_t wbase = su32(st);
+          const uint32_t ihi = su32(st + G::W_BYTES), ilo = su32(st + G::W_BYTES + G::IN_BYTES);
 #pragma unroll 1
-        for (int rr = 0; rr < G::R; rr += 2)
+          for (int t = 0; t < NTAP; ++t) {
+            const int dy = t / 3, dx = t % 3;
+            const uint64_t whi = smem_desc(wbase + (t * 2 + 0) * G::W_TILE, FB * 16);
+            const uint64_t wlo = smem_desc(wbase + (t * 2 + 1) * G::W_TILE, FB * 16);
 #pragma unroll 1
-          for (int cc = 0; cc < TW; cc += 16) {
-            float a[16], b[16];
-            tm_ld16(lane_addr + (uint32_t)(rr * TW + cc), a);
-            tm_ld16(lane_addr + (uint32_t)((rr + 1) * TW + cc), b);
-            tm_wait_ld();
-            store16_pool(p, n, mg, a, b, r0 + rr, c0 + cc);
+            for (int rr = 0; rr < G::R; ++rr) {
+              const uint32_t off = (uint32_t)(((rr + dy) * G::BCOLS + dx) * 16);
+              const uint64_t xh = smem_desc(ihi + off, G::IN_HALF);
+              const uint64_t xl = smem_desc(ilo + off, G::IN_HALF);
+              const uint32_t d = dbase + (uint32_t)(rr * G::SEGC);
+              const uint32_t first = (c == 0 && t == 0) ? 0u : 1u;
+              if (ORI == ORI_FP) {
+                mma_tf32(d, whi, xh, G::IDESC, first);
+                mma_tf32(d, wlo, xh, G::IDESC, 1u);
+                mma_tf32(d, whi, xl, G::IDESC, 1u);
+              } else {
+                mma_tf32(d, xh, whi, G::IDESC, first);
+                mma_tf32(d, xh, wlo, G::IDESC, 1u);
+                mma_tf32(d, xl, whi, G::IDESC, 1u);
+              }
+            }
           }
+          mma_commit(su32(&empty[s]));
+        }
+        if (!okc) break;
+        mma_commit(su32(&acc_full[b]));
       }
+      // every MMA issued by this thread is complete before TMEM is released
+      mma_commit(su32(&done_bar));
+      wait(&done_bar, 0u);
     }
+    __syncwarp();
   } else {
-    // Split over chunks: every CTA publishes its accumulators [m][column] in
-    // shared memory; CTA rank r then reduces the columns with
-    // (column / 16) % ksplit == r over ranks 0..ksplit-1 in order.
-    namespace cg = cooperative_groups;
-    cg::cluster_group cluster = cg::this_cluster();
-    const int rank = (int)cluster.block_rank();
-    float* red = reinterpret_cast<float*>(smem);
-#pragma unroll 1
-    for (int col = 0; col < NCOL; col += 16) {
-      float v[16];
-      tm_ld16(lane_addr + (uint32_t)col, v);
-      tm_wait_ld();
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lane quadrant of this warp
+    const int et = (warp - 5) * 32 + lane;
+    (void)et;
+    const bool pool = p.flags & PP_POOL2;
+    for (int i = 0; i < nmine && !abort_s; ++i) {
+      const int b = i & 1, ub = i >> 1;
+      if (!wait(&acc_full[b], (uint32_t)(ub & 1))) break;
+      tm_fence_after();
+      const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
+      const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NCOL);
+      if (ORI == ORI_FP) {
+        // lane = filter; columns = pixels of row segment rr
+        const int jr = T.fb * FB + 32 * q + lane;
+        const bool valid = jr < p.Co;
+        const int o = valid ? __ldg(p.perm + jr) : 0;
+        const float bs = (valid && p.bias) ? __ldg(p.bias + jr) : 0.f;
+        for (int rr = 0; rr < G::R; rr += (pool ? 2 : 1)) {
+          const int row = T.r0 + rr;
+          for (int cc = 0; cc < TW; cc += 16) {
+            float a[16], bb[16];
+            tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + cc), a);
+            if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + cc), bb);
+            tm_wait_ld();
+            // the TMEM loads above are warp-collective; lanes without an output skip only the stores
+            if (valid && row < p.H) {
+            const int col = T.c0 + cc;
+            const float* sk0 = (p.flags & PP_ADD_SKIP) ? p.skip + (((size_t)T.n * p.Co + o) * p.H + row) * p.W : nullptr;
 #pragma unroll
-      for (int k = 0; k < 16; ++k)  // a CTA with no chunk (or a failed wait) contributes zeros
-        red[(size_t)m * NCOL + ((col + k + m) & (NCOL - 1))] = (ok && cend > cbeg) ? v[k] : 0.f;
-    }
-    cluster.sync();
-    const int cpr = TW / 16;  // 16-column blocks per row
-#pragma unroll 1
-    for (int blk = pool ? 0 : rank; blk < NCOL / 16; blk += pool ? 1 : p.ksplit) {
-      const int rr = blk / cpr, cc = (blk - rr * cpr) * 16;
-      if (pool && ((rr & 1) || ((blk / 2) % p.ksplit) != rank)) continue;
-      float a[16], b[16];
+            for (int k = 0; k < 16; ++k) {
+              a[k] += bs;
+              if (sk0 && col + k < p.W) a[k] += __ldg(sk0 + col + k);
+              if (p.flags & PP_RELU) a[k] = fmaxf(a[k], 0.f);
+            }
+            if (!pool) {
+              float* yo = p.y + (((size_t)T.n * p.Co + o) * p.H + row) * p.W;
+              if (col + 16 <= p.W && (p.W & 3) == 0) {
 #pragma unroll
-      for (int k = 0; k < 16; ++k) a[k] = b[k] = 0.f;
-#pragma unroll 1
-      for (int s2 = 0; s2 < p.ksplit; ++s2) {
-        const float* rem = cluster.map_shared_rank(red, s2) + (size_t)m * NCOL;
+                for (int k = 0; k < 16; k += 4)
+                  *reinterpret_cast<float4*>(yo + col + k) = make_float4(a[k], a[k + 1], a[k + 2], a[k + 3]);
+              } else {
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          a[k] += rem[(blk * 16 + k + m) & (NCOL - 1)];
-          if (pool) b[k] += rem[((blk + cpr) * 16 + k + m) & (NCOL - 1)];
+                for (int k = 0; k < 16; ++k)
+                  if (col + k < p.W) yo[col + k] = a[k];
+              }
+            } else {
+              const float* sk1 = sk0 ? sk0 + p.W : nullptr;
+#pragma unroll
+              for (int k = 0; k < 16; ++k) {
+                bb[k] += bs;
+                if (sk1 && col + k < p.W) bb[k] += __ldg(sk1 + col + k);
+                if (p.flags & PP_RELU) bb[k] = fmaxf(bb[k], 0.f);
+              }
+              const int Ho = p.H / 2, Wo = p.W / 2;
+              float* yo = p.y + (((size_t)T.n * p.Co + o) * Ho + (row >> 1)) * Wo;
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const int pc = (col >> 1) + k;
+                if (pc < Wo) yo[pc] = fmaxf(fmaxf(a[2 * k], a[2 * k + 1]), fmaxf(bb[2 * k], bb[2 * k + 1]));
+              }
+            }
+            }
+          }
+        }
+      } else {
+        // lane = pixel 32q + lane of row segment rr; columns = filters
+        const int col = T.c0 + 32 * q + lane;
+        for (int rr = 0; rr < G::R; rr += (pool ? 2 : 1)) {
+          const int row = T.r0 + rr;
+          for (int jj = 0; jj < FB; jj += 16) {
+            float a[16], bb[16];
+            tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + jj), a);
+            if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + jj), bb);
+            tm_wait_ld();
+#pragma unroll 4
+            for (int k = 0; k < 16; ++k) {
+              const int jr = T.fb * FB + jj + k;
+              if (jr >= p.Co) break;  // uniform across the warp
+              const int o = __ldg(p.perm + jr);
+              const float bs = p.bias ? __ldg(p.bias + jr) : 0.f;
+              float v = a[k] + bs;
+              const size_t plane = ((size_t)T.n * p.Co + o) * p.H;
+              const bool in0 = row < p.H && col < p.W;
+              if ((p.flags & PP_ADD_SKIP) && in0) v += __ldg(p.skip + (plane + row) * p.W + col);
+              if (p.flags & PP_RELU) v = fmaxf(v, 0.f);
+              if (!pool) {
+                if (in0) p.y[(plane + row) * p.W + col] = v;
+              } else {
+                float u = bb[k] + bs;
+                if ((p.flags & PP_ADD_SKIP) && in0) u += __ldg(p.skip + (plane + row + 1) * p.W + col);
+                if (p.flags & PP_RELU) u = fmaxf(u, 0.f);
+                float m = fmaxf(v, u);
+                const float m2 = __shfl_down_sync(0xffffffffu, m, 1);
+                if (((col & 1) == 0) && in0) {
+                  const int Ho = p.H / 2, Wo = p.W / 2;
+                  p.y[(((size_t)T.n * p.Co + o) * Ho + (row >> 1)) * Wo + (col >> 1)] = fmaxf(m, m2);
+                }
+              }
+            }
+          }
         }
       }
-      if (pool)
-        store16_pool(p, n, mg, a, b, r0 + rr, c0 + cc);
-      else
-        store16(p, n, mg, a, r0 + rr, c0 + cc);
+      tm_fence_before();
+      mbar_arrive(su32(&acc_empty[b]));
     }
-    cluster.sync();
   }
 
   tm_fence_before();
   __syncthreads();
   tm_fence_after();
-  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(NCOL));
+  if (warp == MMA_WARP)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(2 * NCOL));
 }
 
-template <int TW>
+template <int ORI, int TW, int FB>
 cudaError_t set_attr() {
-  cudaError_t e = cudaFuncSetAttribute(ppconv_tc_kernel<TW, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Geo<TW>::SMEM_ALLOC);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(ppconv_tc_kernel<TW, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              Geo<TW>::SMEM_ALLOC);
+  return cudaFuncSetAttribute(ppconv_tc_kernel<ORI, TW, FB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              Geo<ORI, TW, FB>::SMEM_ALLOC);
 }
 
 bool g_done[64] = {};
@@ -461,74 +441,65 @@ cudaError_t prepare() {
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 64 && g_done[dev]) return cudaSuccess;
-  if ((e = set_attr<16>()) != cudaSuccess) return e;
-  if ((e = set_attr<32>()) != cudaSuccess) return e;
-  if ((e = set_attr<64>()) != cudaSuccess) return e;
-  if ((e = set_attr<128>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_FP, 16, 128>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_FP, 32, 128>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_FP, 64, 128>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_FP, 128, 128>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_PF, 128, 64>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_PF, 128, 128>()) != cudaSuccess) return e;
   if (dev < 64) g_done[dev] = true;
   return cudaSuccess;
 }
 
-int choose_split(int64_t base_ctas, int nch) {
-  const int64_t slots = 152;  // one CTA per SM
-  int best = 1;
-  double best_t = 1e30;
-  for (int ks = 1; ks <= MAX_SPLIT && ks <= nch; ks *= 2) {
-    const double waves = (double)((base_ctas * ks + slots - 1) / slots);
-    const double t = waves * (double)((nch + ks - 1) / ks) + (ks > 1 ? 1.0 : 0.0);
-    if (t < best_t - 1e-9) {
-      best_t = t;
-      best = ks;
-    }
-  }
-  return best;
-}
-
-template <int TW>
-cudaError_t launch_tw(const TcParams& p0, int N, cudaStream_t stream) {
+template <int ORI, int TW, int FB>
+cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
+  using G = Geo<ORI, TW, FB>;
   TcParams p = p0;
-  using G = Geo<TW>;
   p.tiles_x = (p.W + TW - 1) / TW;
   p.tiles_y = (p.H + G::R - 1) / G::R;
-  const int64_t base = (int64_t)p.tiles_x * p.tiles_y * p.MT * N;
-  const int ks = choose_split(base, p.nch);
-  p.ksplit = ks;
-  p.cpk = (p.nch + ks - 1) / ks;
+  const int64_t nt = (int64_t)p.tiles_x * p.tiles_y * p.nfb * p.N;
+  if (nt > INT32_MAX) return cudaErrorInvalidValue;
+  p.ntiles = (int)nt;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.tiles_x * p.tiles_y, p.MT, N * ks);
+  cfg.gridDim = dim3((unsigned)std::min<int64_t>(nt, sms));
   cfg.blockDim = dim3(NTHREADS);
   cfg.dynamicSmemBytes = G::SMEM_ALLOC;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  if (ks > 1) {
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = ks;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<TW, true>, p);
-  }
-  return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<TW, false>, p);
+  return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB>, p);
 }
+
+int g_sms = 0;
 
 }  // namespace
 
 namespace ppc {
 
-pp_status tc_prepare() { return prepare() == cudaSuccess ? PP_OK : PP_ERR_CUDA; }
+pp_status tc_prepare() {
+  if (prepare() != cudaSuccess) return PP_ERR_CUDA;
+  if (!g_sms) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return PP_ERR_CUDA;
+  }
+  return PP_OK;
+}
 
-// Dense per-tap weights of every (128-filter tile, 8-channel chunk), split into
-// tf32 hi / lo, in the canonical K-major layout: element (filter m, channel k)
-// of a 4 KB tile at byte (k / 4) * 2048 + m * 16 + (k % 4) * 4.
+// Dense per-tap weights of every (FB-filter block, 8-channel chunk), split into
+// tf32 hi / lo, in the canonical K-major layout: element (filter f, channel k)
+// of a tile at byte (k / 4) * (FB * 16) + f * 16 + (k % 4) * 4.  FB = 64 for
+// layers with at most 64 filters, else 128.
 pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
   const int Co = pk->Co, Ci = pk->Ci;
-  T->MT = (Co + TC_M - 1) / TC_M;
+  const int FB = Co <= 64 ? 64 : 128;
+  T->FB = FB;
+  T->nfb = (Co + FB - 1) / FB;
   T->nch = (Ci + KC - 1) / KC;
-  const size_t total = (size_t)T->MT * T->nch * A_BYTES;
+  const size_t wtile = (size_t)FB * KC * 4;
+  const size_t wchunk = NTAP * 2 * wtile;
+  const size_t total = (size_t)T->nfb * T->nch * wchunk;
   std::vector<float> host(total / 4, 0.f);
   for (int j = 0; j < Co; ++j) {
-    const int mt = j / TC_M, m = j % TC_M;
+    const int fb = j / FB, f = j % FB;
     for (int32_t e = pk->kptr[j]; e < pk->kptr[j + 1]; ++e) {
       const int i = pk->kidx[e], c = i / KC, k = i % KC;
       const uint8_t* taps = &pk->taps[4 * pk->kpat[e]];
@@ -541,10 +512,10 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
         std::memcpy(&hi, &bits, 4);
         const float lo = w - hi;
         const int t = taps[s];
-        const size_t base = ((size_t)mt * T->nch + c) * A_BYTES + (size_t)t * 2 * A_TILE;
-        const size_t within = (size_t)(k / 4) * (TC_M * 16) + (size_t)m * 16 + (size_t)(k % 4) * 4;
+        const size_t base = ((size_t)fb * T->nch + c) * wchunk + (size_t)t * 2 * wtile;
+        const size_t within = (size_t)(k / 4) * (FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
         host[(base + within) / 4] = hi;
-        host[(base + A_TILE + within) / 4] = lo;
+        host[(base + wtile + within) / 4] = lo;
       }
     }
   }
@@ -566,15 +537,25 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
   return PP_OK;
 }
 
+// Geometry the launch will use: orientation and tile width for a map width.
+void tc_geometry(const TcLayout& T, int W, int* ori, int* tw) {
+  if (T.FB == 64 || W >= 96) {
+    *ori = ORI_PF;
+    *tw = 128;
+  } else {
+    *ori = ORI_FP;
+    *tw = W <= 16 ? 16 : W <= 32 ? 32 : W <= 64 ? 64 : 128;
+  }
+}
+
 pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N, int H,
                     int W, int flags, cudaStream_t stream) {
-  if ((int64_t)N * MAX_SPLIT > 65535 || T.MT > 65535) return PP_ERR_UNSUPPORTED;
-  if (prepare() != cudaSuccess) return PP_ERR_CUDA;
+  if (tc_prepare() != PP_OK) return PP_ERR_CUDA;
   TcParams p;
   p.x = x;
   p.y = y;
   p.skip = (flags & PP_ADD_SKIP) ? skip : nullptr;
-  p.a = T.a;
+  p.wt = T.a;
   p.perm = M.perm;
   p.bias = M.bias;
   p.status = T.status;
@@ -584,17 +565,22 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
   p.H = H;
   p.W = W;
   p.nch = T.nch;
-  p.MT = T.MT;
+  p.nfb = T.nfb;
+  p.FB = T.FB;
   p.flags = flags;
+  int ori, tw;
+  tc_geometry(T, W, &ori, &tw);
   cudaError_t e;
-  if (W <= 16)
-    e = launch_tw<16>(p, N, stream);
-  else if (W <= 32)
-    e = launch_tw<32>(p, N, stream);
-  else if (W <= 64)
-    e = launch_tw<64>(p, N, stream);
+  if (ori == ORI_PF)
+    e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, g_sms) : launch<ORI_PF, 128, 128>(p, stream, g_sms);
+  else if (tw == 16)
+    e = launch<ORI_FP, 16, 128>(p, stream, g_sms);
+  else if (tw == 32)
+    e = launch<ORI_FP, 32, 128>(p, stream, g_sms);
+  else if (tw == 64)
+    e = launch<ORI_FP, 64, 128>(p, stream, g_sms);
   else
-    e = launch_tw<128>(p, N, stream);
+    e = launch<ORI_FP, 128, 128>(p, stream, g_sms);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return PP_ERR_CUDA;

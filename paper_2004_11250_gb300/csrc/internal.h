@@ -49,7 +49,7 @@ struct TmLayout {
 
 // Dense per-tap tf32 hi/lo weight tiles of the tensor-core kernel (conv_tc.cu).
 struct TcLayout {
-  int MT = 0, nch = 0;
+  int FB = 128, nfb = 0, nch = 0;
   void* dmem = nullptr;
   size_t dbytes = 0;
   const unsigned char* a = nullptr;
