@@ -38,6 +38,7 @@
 // Every wait on an mbarrier is bounded; on timeout the kernel records an error
 // in the layer's device status word and skips the rest of its work.
 #include <cooperative_groups.h>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -52,9 +53,11 @@ namespace {
 constexpr int KC = 8;              // input channels per chunk (MMA K for tf32)
 constexpr int NTAP = 9;
 constexpr int NCOL = 256;          // TMEM columns of one accumulator buffer
-constexpr int NLOAD = 128;         // loader threads (warps 0-3)
-constexpr int MMA_WARP = 4;        // warp 4: TMEM owner and MMA issuer
-constexpr int NTHREADS = 288;      // + epilogue warps 5-8
+constexpr int NLOAD = 256;         // loader threads (warps 0-7)
+constexpr int MMA_WARP = 8;        // warp 8: TMEM owner and MMA issuer
+constexpr int EPI_WARP0 = 9;       // warps 9-12: epilogue, one per TMEM lane quadrant
+constexpr int NTHREADS = 416;
+constexpr int LBATCH = 4;          // loader items whose global loads are in flight together
 constexpr long WAIT_LIMIT = 1L << 22;  // mbarrier polls before a wait gives up
 
 // Orientation of the GEMM on the tensor core.
@@ -74,6 +77,7 @@ struct TcParams {
   int nch, nfb, FB;
   int tiles_x, tiles_y, ntiles;
   int flags;
+  int use_tma;  // input tiles by tensor-map copy (W % 4 == 0, aligned x), else per-thread loads
 };
 
 __device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -108,6 +112,25 @@ __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
 __device__ __forceinline__ void mbar_arrive(uint32_t a) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
 }
+// Add an expected transaction count without arriving.
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+// Named barrier over the loader warps only.  Every loader thread reaches each
+// use of it: loop exits are decided together with loader_any.
+__device__ __forceinline__ void loader_sync() { asm volatile("bar.sync 1, %0;" ::"n"(NLOAD) : "memory"); }
+// OR of v over the loader threads (a barrier too), so all of them take the same branch.
+__device__ __forceinline__ bool loader_any(bool v) {
+  uint32_t r;
+  asm volatile("{ .reg .pred p, q; setp.ne.u32 p, %1, 0; bar.red.or.pred q, 1, %2, p; selp.u32 %0, 1, 0, q; }"
+               : "=r"(r)
+               : "r"((uint32_t)v), "n"(NLOAD)
+               : "memory");
+  return r != 0;
+}
 
 __device__ __forceinline__ void tm_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tm_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -139,10 +162,15 @@ struct Geo {
   static constexpr int NPIX = BROWS * BCOLS;              // staged input pixels
   static constexpr int IN_HALF = NPIX * 16;               // one K half (4 channels) of hi or lo
   static constexpr int IN_BYTES = 2 * IN_HALF;            // hi or lo, 8 channels
+  static constexpr int RAW_W = TW + 8;                    // tensor-map box width: columns c0-4 .. c0+TW+3
+  static constexpr int RAW = KC * BROWS * RAW_W * 4;      // box [8 channels][BROWS][RAW_W], landed in the lo area
+  static constexpr int LO_BYTES = IN_BYTES > RAW ? IN_BYTES : RAW;
   static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo
   static constexpr int W_BYTES = NTAP * 2 * W_TILE;       // weights of one chunk
-  static constexpr int STAGE = W_BYTES + 2 * IN_BYTES;
+  static constexpr int STAGE = W_BYTES + IN_BYTES + LO_BYTES;
   static constexpr int SMEM_ALLOC = 2 * STAGE + 1024;
+  static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
+  static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
   static constexpr uint32_t IDESC = ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB);
 };
 
@@ -163,11 +191,11 @@ __device__ __forceinline__ Tile tile_of(const TcParams& p, int t, int R, int TW)
 }
 
 template <int ORI, int TW, int FB>
-__global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p) {
+__global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p, const __grid_constant__ CUtensorMap xmap) {
   using G = Geo<ORI, TW, FB>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
+  __shared__ __align__(8) uint64_t full[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
 
@@ -191,6 +219,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
       mbar_init(su32(&acc_empty[s]), 128);
+      mbar_init(su32(&raw_full[s]), 1);
     }
     mbar_init(su32(&done_bar), 1);
     abort_s = 0;
@@ -207,57 +236,111 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
   const uint32_t tmem = tmem_s;
   const int nmine = p.ntiles > (int)blockIdx.x ? (p.ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
-  if (warp < 4) {
+  if (warp < MMA_WARP) {
     // ------------------------------------------------------------ loaders
     int g = 0;  // chunk sequence number of this CTA
-    for (int i = 0; i < nmine && !abort_s; ++i) {
+    bool stop = false;  // identical in every loader thread (decided by loader_any)
+    for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
       for (int c = 0; c < p.nch; ++c, ++g) {
         const int s = g & 1, use = g >> 1;
-        if (use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1))) break;
+        if (loader_any(use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1)))) {
+          stop = true;
+          break;
+        }
         unsigned char* st = smem + s * G::STAGE;
+        float4* hi = reinterpret_cast<float4*>(st + G::W_BYTES);
+        float4* lo = reinterpret_cast<float4*>(st + G::W_BYTES + G::IN_BYTES);
         if (tid == 0) {
+          // weights: one bulk copy counted on full[s] (thread 0 arrives later, after its own stores)
           const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * G::W_BYTES;
-          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(&full[s])),
-                       "r"(G::W_BYTES)
-                       : "memory");
+          mbar_expect_tx(su32(&full[s]), G::W_BYTES);
           asm volatile(
               "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                   su32(st)),
               "l"(src), "r"(G::W_BYTES), "r"(su32(&full[s]))
               : "memory");
-        }
-        // input tile: item = (K half, pixel); 4 channels of one pixel, split into hi / lo
-        float4* hi = reinterpret_cast<float4*>(st + G::W_BYTES);
-        float4* lo = reinterpret_cast<float4*>(st + G::W_BYTES + G::IN_BYTES);
-        const int ch0 = c * KC;
-        for (int it = tid; it < 2 * G::NPIX; it += NLOAD) {
-          const int kh = it >= G::NPIX ? 1 : 0;
-          const int pix = it - kh * G::NPIX;
-          const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
-          const int r = T.r0 - 1 + br, cc = T.c0 - 1 + bc;
-          float v[4];
-          const bool inside = (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const int ch = ch0 + kh * 4 + k;
-            v[k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
+          if (p.use_tma) {
+            // raw input box [8 channels][rows r0-1 ..][columns c0-4 ..] into the lo area; outside the
+            // image the copy fills zeros, which is the convolution's zero padding
+            mbar_arrive_expect_tx(su32(&raw_full[s]), G::RAW);
+            asm volatile(
+                "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+                "%4, %5}], [%6];" ::"r"(su32(lo)),
+                "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(T.c0 - 4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
+                "r"(su32(&raw_full[s]))
+                : "memory");
           }
-          float4 h, l;
-          h.x = __uint_as_float(__float_as_uint(v[0]) & 0xFFFFE000u);
-          h.y = __uint_as_float(__float_as_uint(v[1]) & 0xFFFFE000u);
-          h.z = __uint_as_float(__float_as_uint(v[2]) & 0xFFFFE000u);
-          h.w = __uint_as_float(__float_as_uint(v[3]) & 0xFFFFE000u);
-          l = make_float4(v[0] - h.x, v[1] - h.y, v[2] - h.z, v[3] - h.w);
-          hi[it] = h;
-          lo[it] = l;
+        }
+        const int ch0 = c * KC;
+        if (p.use_tma) {
+          if (loader_any(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
+            stop = true;
+            break;
+          }
+          const float* raw = reinterpret_cast<const float*>(lo);
+          float v[G::ITEMS][4];
+#pragma unroll
+          for (int b = 0; b < G::ITEMS; ++b) {
+            const int it = b * NLOAD + tid;
+            const int kh = it >= G::NPIX ? 1 : 0;
+            const int pix = it - kh * G::NPIX;
+            const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              v[b][k] = it < 2 * G::NPIX ? raw[((kh * 4 + k) * G::BROWS + br) * G::RAW_W + bc + 3] : 0.f;
+          }
+          loader_sync();  // every raw value is in registers before the lo area is rewritten
+#pragma unroll
+          for (int b = 0; b < G::ITEMS; ++b) {
+            const int it = b * NLOAD + tid;
+            if (it < 2 * G::NPIX) {
+              float4 h;
+              h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
+              h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
+              h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
+              h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
+              hi[it] = h;
+              lo[it] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+            }
+          }
+        } else {
+        // Items in batches of LBATCH per thread: all global loads of a batch are
+        // issued before any is used, so their latencies overlap.
+        for (int base = 0; base < 2 * G::NPIX; base += NLOAD * LBATCH) {
+          float v[LBATCH][4];
+#pragma unroll
+          for (int b = 0; b < LBATCH; ++b) {
+            const int it = base + b * NLOAD + tid;
+            const int kh = it >= G::NPIX ? 1 : 0;
+            const int pix = it - kh * G::NPIX;
+            const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
+            const int r = T.r0 - 1 + br, cc = T.c0 - 1 + bc;
+            const bool inside = it < 2 * G::NPIX && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int ch = ch0 + kh * 4 + k;
+              v[b][k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
+            }
+          }
+#pragma unroll
+          for (int b = 0; b < LBATCH; ++b) {
+            const int it = base + b * NLOAD + tid;
+            if (it < 2 * G::NPIX) {
+              float4 h;
+              h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
+              h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
+              h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
+              h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
+              hi[it] = h;
+              lo[it] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+            }
+          }
+        }
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        if (tid == 0)
-          ;  // thread 0 arrived with the transaction count above
-        else
-          mbar_arrive(su32(&full[s]));
+        mbar_arrive(su32(&full[s]));
       }
     }
   } else if (warp == MMA_WARP) {
@@ -315,13 +398,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;  // TMEM lane quadrant of this warp
-    const int et = (warp - 5) * 32 + lane;
-    (void)et;
+    const int q = warp & 3;  // TMEM lane quadrant of this warp (warps 9-12 -> 1, 2, 3, 0)
     const bool pool = p.flags & PP_POOL2;
-    for (int i = 0; i < nmine && !abort_s; ++i) {
+    for (int i = 0; i < nmine; ++i) {
       const int b = i & 1, ub = i >> 1;
-      if (!wait(&acc_full[b], (uint32_t)(ub & 1))) break;
+      // the whole warp leaves together: its TMEM loads and shuffles are warp-collective
+      if (!__all_sync(0xffffffffu, wait(&acc_full[b], (uint32_t)(ub & 1)))) break;
       tm_fence_after();
       const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
       const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NCOL);
@@ -451,12 +533,34 @@ cudaError_t prepare() {
   return cudaSuccess;
 }
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn g_encode = nullptr;
+
+// 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][8][R+2][TW+8].
+template <int ORI, int TW, int FB>
+bool make_xmap(CUtensorMap* m, const TcParams& p) {
+  using G = Geo<ORI, TW, FB>;
+  if (!g_encode) return false;
+  const cuuint64_t dims[4] = {(cuuint64_t)p.W, (cuuint64_t)p.H, (cuuint64_t)p.Ci, (cuuint64_t)p.N};
+  const cuuint64_t strides[3] = {(cuuint64_t)p.W * 4, (cuuint64_t)p.W * p.H * 4, (cuuint64_t)p.W * p.H * p.Ci * 4};
+  const cuuint32_t box[4] = {(cuuint32_t)G::RAW_W, (cuuint32_t)G::BROWS, (cuuint32_t)KC, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(p.x), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int ORI, int TW, int FB>
 cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
   using G = Geo<ORI, TW, FB>;
   TcParams p = p0;
   p.tiles_x = (p.W + TW - 1) / TW;
   p.tiles_y = (p.H + G::R - 1) / G::R;
+  CUtensorMap xmap;
+  std::memset(&xmap, 0, sizeof(xmap));
+  p.use_tma = ((p.W & 3) == 0 && (reinterpret_cast<uintptr_t>(p.x) & 15) == 0 && make_xmap<ORI, TW, FB>(&xmap, p)) ? 1 : 0;
   const int64_t nt = (int64_t)p.tiles_x * p.tiles_y * p.nfb * p.N;
   if (nt > INT32_MAX) return cudaErrorInvalidValue;
   p.ntiles = (int)nt;
@@ -465,7 +569,7 @@ cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
   cfg.blockDim = dim3(NTHREADS);
   cfg.dynamicSmemBytes = G::SMEM_ALLOC;
   cfg.stream = stream;
-  return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB>, p);
+  return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB>, p, xmap);
 }
 
 int g_sms = 0;
@@ -476,6 +580,15 @@ namespace ppc {
 
 pp_status tc_prepare() {
   if (prepare() != cudaSuccess) return PP_ERR_CUDA;
+  if (!g_encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+    else
+      cudaGetLastError();  // without the entry point every launch uses per-thread loads
+  }
   if (!g_sms) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
