@@ -163,6 +163,15 @@ pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const
 pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
 /* The kernel that pp_conv_forward will run (PP_KERNEL_TC, _TMEM or _REGISTER). */
 pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
+/* Time every kernel that can run this layer on zero-filled scratch tensors of
+ * the given shape and flags (a few launches each, on stream, synchronous) and
+ * keep the fastest for the layer.  The kernels differ in speed by layer shape:
+ * the tensor-core kernel needs many output tiles to fill the GPU, the FMA
+ * kernels split small layers across thread-block clusters.  Allocates and
+ * frees scratch device memory; must not be called during stream capture.
+ * Errors: PP_ERR_INVALID_ARG, PP_ERR_UNSUPPORTED, PP_ERR_CUDA, PP_ERR_OOM. */
+pp_status pp_layer_autotune(pp_layer* layer, int N, int H, int W, int flags, void* stream);
+
 /* Synchronous: *device_error = 0 unless a kernel of this layer gave up a
  * bounded wait (its output is then invalid); the word is cleared by the read. */
 pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);
@@ -205,7 +214,9 @@ pp_status pp_net_add_conv(pp_net* net, const pp_layer* layer, int flags, int ski
 pp_status pp_net_add_dense(pp_net* net, const pp_dense* layer, int flags, int skip_from);
 
 /* Plan activation buffers and allocate them on the current device (library
- * owned).  Must be called once, after the last add and before the first run. */
+ * owned), then autotune the kernel of every pruned op at its shape
+ * (pp_layer_autotune; this changes the kernel choice of the borrowed layers).
+ * Must be called once, after the last add and before the first run. */
 pp_status pp_net_finalize(pp_net* net);
 
 /* Shape of the network output (any pointer may be NULL). */

@@ -700,6 +700,68 @@ extern "C" pp_status pp_layer_kernel(const pp_layer* L, int* kernel) {
   return PP_OK;
 }
 
+extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int flags, void* stream_) {
+  if (!L || N < 1 || H < 1 || W < 1) return PP_ERR_INVALID_ARG;
+  if (flags & ~(PP_ADD_SKIP | PP_RELU | PP_POOL2)) return PP_ERR_INVALID_ARG;
+  if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  std::vector<int> cand;
+  if (L->tc_ok) cand.push_back(PP_KERNEL_TC);
+  if (L->tm_ok) cand.push_back(PP_KERNEL_TMEM);
+  if (cand.empty()) cand.push_back(PP_KERNEL_REGISTER);
+  if (cand.size() == 1) {
+    L->kernel = cand[0];
+    return PP_OK;
+  }
+  const size_t in_elems = (size_t)N * L->Ci * H * W, out_elems = (size_t)N * L->Co * H * W;
+  float *x = nullptr, *y = nullptr, *sk = nullptr;
+  if (cudaMalloc(&x, in_elems * 4) != cudaSuccess || cudaMalloc(&y, out_elems * 4) != cudaSuccess ||
+      ((flags & PP_ADD_SKIP) && cudaMalloc(&sk, out_elems * 4) != cudaSuccess)) {
+    cudaGetLastError();
+    cudaFree(x);
+    cudaFree(y);
+    return PP_ERR_OOM;
+  }
+  pp_status st = PP_OK;
+  if (cudaMemsetAsync(x, 0, in_elems * 4, stream) != cudaSuccess ||
+      (sk && cudaMemsetAsync(sk, 0, out_elems * 4, stream) != cudaSuccess))
+    st = PP_ERR_CUDA;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (st == PP_OK && (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess)) st = PP_ERR_CUDA;
+  const int saved = L->kernel;
+  int best = saved;
+  float best_ms = 1e30f;
+  for (int k : cand) {
+    if (st != PP_OK) break;
+    L->kernel = k;
+    for (int w = 0; w < 2 && st == PP_OK; ++w) st = launch(L, x, y, sk, N, H, W, flags, stream);
+    if (st != PP_OK) break;
+    if (cudaEventRecord(e0, stream) != cudaSuccess) {
+      st = PP_ERR_CUDA;
+      break;
+    }
+    for (int r = 0; r < 5 && st == PP_OK; ++r) st = launch(L, x, y, sk, N, H, W, flags, stream);
+    float ms = 0.f;
+    if (st != PP_OK || cudaEventRecord(e1, stream) != cudaSuccess || cudaEventSynchronize(e1) != cudaSuccess ||
+        cudaEventElapsedTime(&ms, e0, e1) != cudaSuccess) {
+      st = st != PP_OK ? st : PP_ERR_CUDA;
+      break;
+    }
+    if (ms < best_ms) {
+      best_ms = ms;
+      best = k;
+    }
+  }
+  L->kernel = st == PP_OK ? best : saved;
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  cudaStreamSynchronize(stream);
+  cudaFree(x);
+  cudaFree(y);
+  cudaFree(sk);
+  return st;
+}
+
 extern "C" pp_status pp_layer_device_status(const pp_layer* L, int* device_error) {
   if (!L || !device_error) return PP_ERR_INVALID_ARG;
   *device_error = 0;

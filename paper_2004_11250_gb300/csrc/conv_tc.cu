@@ -361,26 +361,28 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           }
           tm_fence_after();
           const unsigned char* st = smem + s * G::STAGE;
-          const uint32_t wbase = su32(st);
-          const uint32_t ihi = su32(st + G::W_BYTES), ilo = su32(st + G::W_BYTES + G::IN_BYTES);
-#pragma unroll 1
+          // Descriptors hold address / 16 in their low 14 bits and every operand
+          // lies below 256 KB, so moving an operand is one add to the descriptor.
+          const uint64_t w0 = smem_desc(su32(st), FB * 16);
+          const uint64_t xh0 = smem_desc(su32(st + G::W_BYTES), G::IN_HALF);
+          const uint64_t xl0 = smem_desc(su32(st + G::W_BYTES + G::IN_HALF * 2), G::IN_HALF);
+          const uint32_t acc0 = c == 0 ? 0u : 1u;  // the tile's first chunk overwrites the accumulators
+#pragma unroll
           for (int t = 0; t < NTAP; ++t) {
             const int dy = t / 3, dx = t % 3;
-            const uint64_t whi = smem_desc(wbase + (t * 2 + 0) * G::W_TILE, FB * 16);
-            const uint64_t wlo = smem_desc(wbase + (t * 2 + 1) * G::W_TILE, FB * 16);
-#pragma unroll 1
+            const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * G::W_TILE / 16);
+            const uint64_t wlo = w0 + (uint64_t)((t * 2 + 1) * G::W_TILE / 16);
+#pragma unroll(G::R <= 8 ? G::R : 4)
             for (int rr = 0; rr < G::R; ++rr) {
-              const uint32_t off = (uint32_t)(((rr + dy) * G::BCOLS + dx) * 16);
-              const uint64_t xh = smem_desc(ihi + off, G::IN_HALF);
-              const uint64_t xl = smem_desc(ilo + off, G::IN_HALF);
+              const uint64_t off = (uint64_t)((rr + dy) * G::BCOLS + dx);  // pixels of 16 bytes
+              const uint64_t xh = xh0 + off, xl = xl0 + off;
               const uint32_t d = dbase + (uint32_t)(rr * G::SEGC);
-              const uint32_t first = (c == 0 && t == 0) ? 0u : 1u;
               if (ORI == ORI_FP) {
-                mma_tf32(d, whi, xh, G::IDESC, first);
+                mma_tf32(d, whi, xh, G::IDESC, t == 0 ? acc0 : 1u);
                 mma_tf32(d, wlo, xh, G::IDESC, 1u);
                 mma_tf32(d, whi, xl, G::IDESC, 1u);
               } else {
-                mma_tf32(d, xh, whi, G::IDESC, first);
+                mma_tf32(d, xh, whi, G::IDESC, t == 0 ? acc0 : 1u);
                 mma_tf32(d, xh, wlo, G::IDESC, 1u);
                 mma_tf32(d, xl, whi, G::IDESC, 1u);
               }
@@ -470,7 +472,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + jj), a);
             if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + jj), bb);
             tm_wait_ld();
-#pragma unroll 4
+#pragma unroll
             for (int k = 0; k < 16; ++k) {
               const int jr = T.fb * FB + jj + k;
               if (jr >= p.Co) break;  // uniform across the warp

@@ -187,6 +187,16 @@ extern "C" pp_status pp_net_finalize(pp_net* net) {
     }
     net->buffers.push_back(p);
   }
+  // Pick each pruned op's kernel at the op's own shape.
+  for (const OpDesc& d : net->ops) {
+    if (!d.conv) continue;
+    pp_status st = pp_layer_autotune(const_cast<pp_layer*>(d.conv), net->N, d.H, d.W, d.flags, nullptr);
+    if (st != PP_OK) {
+      for (float* q : net->buffers) cudaFree(q);
+      net->buffers.clear();
+      return st;
+    }
+  }
   net->finalized = true;
   return PP_OK;
 }

@@ -61,6 +61,7 @@ _SIGS = {
     "pp_layer_set_kernel": ([_P, _I], _I),
     "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_device_status": ([_P, _P], _I),
+    "pp_layer_autotune": ([_P, _I, _I, _I, _I, _P], _I),
     "pp_layer_destroy": ([_P], None),
     "pp_dense_create": ([_P, _P, _I, _I, _P, _PP], _I),
     "pp_dense_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
@@ -215,6 +216,10 @@ def pp_layer_kernel(layer) -> int:
     k = _I()
     _check(lib.pp_layer_kernel(layer, ctypes.byref(k)), "pp_layer_kernel")
     return k.value
+
+
+def pp_layer_autotune(layer, N, H, W, flags, stream=None):
+    _check(lib.pp_layer_autotune(layer, N, H, W, flags, _stream(stream)), "pp_layer_autotune")
 
 
 def pp_layer_device_status(layer) -> int:

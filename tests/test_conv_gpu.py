@@ -130,6 +130,24 @@ def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
         check_within(g, y, s, f"tensor-core kernel {(N, Ci, Co, H, W)}")
 
 
+def test_autotune_keeps_parity(pp, runner, oracle_mod):
+    rng = np.random.default_rng(44)
+    L = synth.small_random_layer(rng, 96, 64, P=8, keep=0.4)
+    x = rng.uniform(-1, 1, (1, 64, 24, 40)).astype(np.float32)
+    dl = runner.DeviceLayer(L)
+    try:
+        pp.pp_layer_autotune(dl.handle, 1, 24, 40, pp.PP_RELU, None)
+        assert pp.pp_layer_kernel(dl.handle) in (pp.PP_KERNEL_TC, pp.PP_KERNEL_TMEM)
+        y = torch.empty((1, 96, 24, 40), device="cuda")
+        dl.forward(dev(x), y, None, 1, 24, 40, pp.PP_RELU, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        yr, s = oracle_layer_full(oracle_mod, L, x, None, True, False)
+        check_within(y.cpu().numpy(), yr, s, "autotuned layer")
+        assert pp.pp_layer_device_status(dl.handle) == 0
+    finally:
+        dl.close()
+
+
 def test_kernel_selection(pp, runner):
     rng = np.random.default_rng(2)
     ring = runner.DeviceLayer(synth.small_random_layer(rng, 8, 8, ring=True))
