@@ -167,8 +167,14 @@ struct Geo {
   static constexpr int LO_BYTES = IN_BYTES > RAW ? IN_BYTES : RAW;
   static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo
   static constexpr int W_BYTES = NTAP * 2 * W_TILE;       // weights of one chunk
-  static constexpr int STAGE = W_BYTES + IN_BYTES + LO_BYTES;
-  static constexpr int SMEM_ALLOC = 2 * STAGE + 1024;
+  // SEP: the raw boxes get a ring of their own (two slots), so the copy for a
+  // chunk can start two chunks ahead instead of waiting for the MMAs that read
+  // the stage; used whenever it fits in shared memory.
+  static constexpr int STAGE_SEP = W_BYTES + 2 * IN_BYTES;
+  static constexpr bool SEP = 2 * STAGE_SEP + 2 * RAW + 1024 <= 232448;
+  static constexpr int STAGE = SEP ? STAGE_SEP : W_BYTES + IN_BYTES + LO_BYTES;
+  static constexpr int RAW_OFF = 2 * STAGE;               // raw slots (SEP)
+  static constexpr int SMEM_ALLOC = 2 * STAGE + (SEP ? 2 * RAW : 0) + 1024;
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
   static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
   static constexpr uint32_t IDESC = ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB);
@@ -195,7 +201,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
   using G = Geo<ORI, TW, FB>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t full[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
+  __shared__ __align__(8) uint64_t full[2], wfull[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
 
@@ -220,6 +226,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       mbar_init(su32(&acc_full[s]), 1);
       mbar_init(su32(&acc_empty[s]), 128);
       mbar_init(su32(&raw_full[s]), 1);
+      mbar_init(su32(&wfull[s]), 1);
     }
     mbar_init(su32(&done_bar), 1);
     abort_s = 0;
@@ -238,6 +245,26 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 
   if (warp < MMA_WARP) {
     // ------------------------------------------------------------ loaders
+    // Thread 0 issues the copies: weights (bulk, on wfull[s]) and, with a tensor
+    // map, the raw input box (on raw_full); all loader threads then transpose the
+    // box into the hi / lo operand tiles and arrive on full[s].
+    const int nall = nmine * p.nch;  // chunks of this CTA
+    auto issue_raw = [&](int gg, unsigned char* dst) {  // thread 0 only
+      const int i = gg / p.nch, c = gg - i * p.nch;
+      const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
+      // box [8 channels][rows r0-1 ..][columns c0-4 ..]; outside the image the
+      // copy fills zeros, which is the convolution's zero padding
+      mbar_arrive_expect_tx(su32(&raw_full[gg & 1]), G::RAW);
+      asm volatile(
+          "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+          "%4, %5}], [%6];" ::"r"(su32(dst)),
+          "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(T.c0 - 4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
+          "r"(su32(&raw_full[gg & 1]))
+          : "memory");
+    };
+    int raw_issued = 0, w_issued = 0;  // thread 0's counts of issued copies
+    if (tid == 0 && p.use_tma && G::SEP)
+      for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + G::RAW_OFF + raw_issued * G::RAW);
     int g = 0;  // chunk sequence number of this CTA
     bool stop = false;  // identical in every loader thread (decided by loader_any)
     for (int i = 0; i < nmine && !stop; ++i) {
@@ -253,33 +280,27 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         float4* hi = reinterpret_cast<float4*>(st + G::W_BYTES);
         float4* lo = reinterpret_cast<float4*>(st + G::W_BYTES + G::IN_BYTES);
         if (tid == 0) {
-          // weights: one bulk copy counted on full[s] (thread 0 arrives later, after its own stores)
           const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * G::W_BYTES;
-          mbar_expect_tx(su32(&full[s]), G::W_BYTES);
+          mbar_arrive_expect_tx(su32(&wfull[s]), G::W_BYTES);
           asm volatile(
               "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                   su32(st)),
-              "l"(src), "r"(G::W_BYTES), "r"(su32(&full[s]))
+              "l"(src), "r"(G::W_BYTES), "r"(su32(&wfull[s]))
               : "memory");
-          if (p.use_tma) {
-            // raw input box [8 channels][rows r0-1 ..][columns c0-4 ..] into the lo area; outside the
-            // image the copy fills zeros, which is the convolution's zero padding
-            mbar_arrive_expect_tx(su32(&raw_full[s]), G::RAW);
-            asm volatile(
-                "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
-                "%4, %5}], [%6];" ::"r"(su32(lo)),
-                "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(T.c0 - 4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
-                "r"(su32(&raw_full[s]))
-                : "memory");
+          ++w_issued;
+          if (p.use_tma && !G::SEP) {
+            issue_raw(g, reinterpret_cast<unsigned char*>(lo));
+            ++raw_issued;
           }
         }
         const int ch0 = c * KC;
         if (p.use_tma) {
-          if (loader_any(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
+          if (loader_any(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
             stop = true;
             break;
           }
-          const float* raw = reinterpret_cast<const float*>(lo);
+          const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g & 1) * G::RAW)
+                                    : reinterpret_cast<const float*>(lo);
           float v[G::ITEMS][4];
 #pragma unroll
           for (int b = 0; b < G::ITEMS; ++b) {
@@ -291,7 +312,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             for (int k = 0; k < 4; ++k)
               v[b][k] = it < 2 * G::NPIX ? raw[((kh * 4 + k) * G::BROWS + br) * G::RAW_W + bc + 3] : 0.f;
           }
-          loader_sync();  // every raw value is in registers before the lo area is rewritten
+          loader_sync();  // every raw value is in registers before its slot is reused
+          if (G::SEP && tid == 0 && raw_issued < nall && raw_issued == g + 2) {
+            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued & 1) * G::RAW);
+            ++raw_issued;
+          }
 #pragma unroll
           for (int b = 0; b < G::ITEMS; ++b) {
             const int it = b * NLOAD + tid;
@@ -306,42 +331,54 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             }
           }
         } else {
-        // Items in batches of LBATCH per thread: all global loads of a batch are
-        // issued before any is used, so their latencies overlap.
-        for (int base = 0; base < 2 * G::NPIX; base += NLOAD * LBATCH) {
-          float v[LBATCH][4];
+          // Items in batches of LBATCH per thread: all global loads of a batch
+          // are issued before any is used, so their latencies overlap.
+          for (int base = 0; base < 2 * G::NPIX; base += NLOAD * LBATCH) {
+            float v[LBATCH][4];
 #pragma unroll
-          for (int b = 0; b < LBATCH; ++b) {
-            const int it = base + b * NLOAD + tid;
-            const int kh = it >= G::NPIX ? 1 : 0;
-            const int pix = it - kh * G::NPIX;
-            const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
-            const int r = T.r0 - 1 + br, cc = T.c0 - 1 + bc;
-            const bool inside = it < 2 * G::NPIX && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
+            for (int b = 0; b < LBATCH; ++b) {
+              const int it = base + b * NLOAD + tid;
+              const int kh = it >= G::NPIX ? 1 : 0;
+              const int pix = it - kh * G::NPIX;
+              const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
+              const int r = T.r0 - 1 + br, cc = T.c0 - 1 + bc;
+              const bool inside = it < 2 * G::NPIX && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const int ch = ch0 + kh * 4 + k;
-              v[b][k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
+              for (int k = 0; k < 4; ++k) {
+                const int ch = ch0 + kh * 4 + k;
+                v[b][k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
+              }
+            }
+#pragma unroll
+            for (int b = 0; b < LBATCH; ++b) {
+              const int it = base + b * NLOAD + tid;
+              if (it < 2 * G::NPIX) {
+                float4 h;
+                h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
+                h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
+                h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
+                h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
+                hi[it] = h;
+                lo[it] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+              }
             }
           }
-#pragma unroll
-          for (int b = 0; b < LBATCH; ++b) {
-            const int it = base + b * NLOAD + tid;
-            if (it < 2 * G::NPIX) {
-              float4 h;
-              h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
-              h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
-              h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
-              h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
-              hi[it] = h;
-              lo[it] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
-            }
-          }
-        }
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         mbar_arrive(su32(&full[s]));
       }
+    }
+    if (tid == 0) {
+      // No copy may still be writing shared memory when the CTA exits: after an
+      // early stop, wait (bounded) for the last copies of each kind to land.
+      for (int gg = raw_issued - 2; gg < raw_issued; ++gg)
+        if (gg >= 0)
+          for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&raw_full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+          }
+      for (int gg = w_issued - 2; gg < w_issued; ++gg)
+        if (gg >= 0)
+          for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&wfull[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+          }
     }
   } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
@@ -355,7 +392,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         bool okc = true;
         for (int c = 0; c < p.nch; ++c, ++g) {
           const int s = g & 1, use = g >> 1;
-          if (!wait(&full[s], (uint32_t)(use & 1))) {
+          if (!wait(&full[s], (uint32_t)(use & 1)) || !wait(&wfull[s], (uint32_t)(use & 1))) {
             okc = false;
             break;
           }
