@@ -559,8 +559,14 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
     M.Ci = L->Ci;
     M.perm = L->perm;
     M.bias = L->has_bias ? L->bias : nullptr;
-    return L->kernel == PP_KERNEL_TC ? ppc::tc_launch(L->tc, M, x, y, skip, N, H, W, flags, stream)
-                                     : ppc::tm_launch(L->tm, M, x, y, skip, N, H, W, flags, stream);
+    if (L->kernel == PP_KERNEL_TC) {
+      const pp_status st = ppc::tc_launch(L->tc, M, x, y, skip, N, H, W, flags, stream);
+      if (st != PP_ERR_UNSUPPORTED) return st;
+      // shapes beyond the tensor-core kernel's 32-bit offsets run on an FMA kernel
+      if (L->tm_ok) return ppc::tm_launch(L->tm, M, x, y, skip, N, H, W, flags, stream);
+    } else {
+      return ppc::tm_launch(L->tm, M, x, y, skip, N, H, W, flags, stream);
+    }
   }
   const int tiles_y = (H + TH - 1) / TH, tiles_x = (W + TW - 1) / TW;
   if ((int64_t)tiles_y * tiles_x > INT32_MAX) return PP_ERR_UNSUPPORTED;

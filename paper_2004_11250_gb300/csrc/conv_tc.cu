@@ -55,8 +55,9 @@ constexpr int NTAP = 9;
 constexpr int NCOL = 256;          // TMEM columns of one accumulator buffer
 constexpr int NLOAD = 256;         // loader threads (warps 0-7)
 constexpr int MMA_WARP = 8;        // warp 8: TMEM owner and MMA issuer
-constexpr int EPI_WARP0 = 9;       // warps 9-12: epilogue, one per TMEM lane quadrant
-constexpr int NTHREADS = 416;
+constexpr int EPI_WARP0 = 9;       // warps 9-16: epilogue, two per TMEM lane quadrant
+constexpr int NEPI = 256;          // epilogue threads
+constexpr int NTHREADS = 544;
 constexpr int LBATCH = 4;          // loader items whose global loads are in flight together
 constexpr long WAIT_LIMIT = 1L << 22;  // mbarrier polls before a wait gives up
 
@@ -224,7 +225,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       mbar_init(su32(&full[s]), NLOAD);
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
-      mbar_init(su32(&acc_empty[s]), 128);
+      mbar_init(su32(&acc_empty[s]), NEPI);
       mbar_init(su32(&raw_full[s]), 1);
       mbar_init(su32(&wfull[s]), 1);
     }
@@ -312,6 +313,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             for (int k = 0; k < 4; ++k)
               v[b][k] = it < 2 * G::NPIX ? raw[((kh * 4 + k) * G::BROWS + br) * G::RAW_W + bc + 3] : 0.f;
           }
+          // The raw slot is rewritten next by a tensor-map copy (async proxy):
+          // each thread orders its generic-proxy reads of the slot before that
+          // copy with a proxy fence, then the loader barrier lets thread 0 issue it.
+          if (G::SEP) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           loader_sync();  // every raw value is in registers before its slot is reused
           if (G::SEP && tid == 0 && raw_issued < nall && raw_issued == g + 2) {
             issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued & 1) * G::RAW);
@@ -437,7 +442,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;  // TMEM lane quadrant of this warp (warps 9-12 -> 1, 2, 3, 0)
+    const int q = warp & 3;                 // TMEM lane quadrant of this warp
+    const int half = (warp - EPI_WARP0) >> 2;  // the two warps of a quadrant split the columns
     const bool pool = p.flags & PP_POOL2;
     for (int i = 0; i < nmine; ++i) {
       const int b = i & 1, ub = i >> 1;
@@ -452,7 +458,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         const bool valid = jr < p.Co;
         const int o = valid ? __ldg(p.perm + jr) : 0;
         const float bs = (valid && p.bias) ? __ldg(p.bias + jr) : 0.f;
-        for (int rr = 0; rr < G::R; rr += (pool ? 2 : 1)) {
+        const int step = pool ? 2 : 1;
+        for (int rr = half * step; rr < G::R; rr += 2 * step) {
           const int row = T.r0 + rr;
           for (int cc = 0; cc < TW; cc += 16) {
             float a[16], bb[16];
@@ -500,38 +507,56 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           }
         }
       } else {
-        // lane = pixel 32q + lane of row segment rr; columns = filters
+        // lane = pixel 32q + lane of row segment rr; columns = filters (this
+        // warp: half of them).  The block's filter indices and biases sit in
+        // registers spread over the lanes (filter j in lane j % 32 of register
+        // j / 32) and are fetched by shuffle; output offsets within an image
+        // fit in 32 bits (checked on the host), so an output costs a shuffle,
+        // a multiply-add and a store.
+        constexpr int NR = FB / 32;
+        int pm[NR];
+        float bv[NR];
+#pragma unroll
+        for (int k = 0; k < NR; ++k) {
+          const int jr = T.fb * FB + 32 * k + lane;
+          pm[k] = jr < p.Co ? __ldg(p.perm + jr) : -1;
+          bv[k] = (jr < p.Co && p.bias) ? __ldg(p.bias + jr) : 0.f;
+        }
         const int col = T.c0 + 32 * q + lane;
+        const int Ho = p.H / 2, Wo = p.W / 2;
+        const int HW = p.H * p.W, HWo = Ho * Wo;
+        const size_t nco = (size_t)T.n * p.Co;
+        float* ybase = p.y + nco * (size_t)(pool ? HWo : HW);
+        const float* sbase = (p.flags & PP_ADD_SKIP) ? p.skip + nco * (size_t)HW : nullptr;
         for (int rr = 0; rr < G::R; rr += (pool ? 2 : 1)) {
           const int row = T.r0 + rr;
-          for (int jj = 0; jj < FB; jj += 16) {
+          const bool in0 = row < p.H && col < p.W;
+          const int roff = row * p.W + col;
+          const int poff = (row >> 1) * Wo + (col >> 1);
+#pragma unroll
+          for (int jj = half * (FB / 2); jj < (half + 1) * (FB / 2); jj += 16) {
             float a[16], bb[16];
             tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + jj), a);
             if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + jj), bb);
             tm_wait_ld();
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
-              const int jr = T.fb * FB + jj + k;
-              if (jr >= p.Co) break;  // uniform across the warp
-              const int o = __ldg(p.perm + jr);
-              const float bs = p.bias ? __ldg(p.bias + jr) : 0.f;
+              const int j = jj + k;
+              const int o = __shfl_sync(0xffffffffu, pm[j >> 5], j & 31);
+              const float bs = __shfl_sync(0xffffffffu, bv[j >> 5], j & 31);
+              if (o < 0) continue;  // past the last filter: the same for every lane
               float v = a[k] + bs;
-              const size_t plane = ((size_t)T.n * p.Co + o) * p.H;
-              const bool in0 = row < p.H && col < p.W;
-              if ((p.flags & PP_ADD_SKIP) && in0) v += __ldg(p.skip + (plane + row) * p.W + col);
+              if (sbase && in0) v += __ldg(sbase + o * HW + roff);
               if (p.flags & PP_RELU) v = fmaxf(v, 0.f);
               if (!pool) {
-                if (in0) p.y[(plane + row) * p.W + col] = v;
+                if (in0) ybase[o * HW + roff] = v;
               } else {
                 float u = bb[k] + bs;
-                if ((p.flags & PP_ADD_SKIP) && in0) u += __ldg(p.skip + (plane + row + 1) * p.W + col);
+                if (sbase && in0) u += __ldg(sbase + o * HW + roff + p.W);
                 if (p.flags & PP_RELU) u = fmaxf(u, 0.f);
-                float m = fmaxf(v, u);
+                const float m = fmaxf(v, u);
                 const float m2 = __shfl_down_sync(0xffffffffu, m, 1);
-                if (((col & 1) == 0) && in0) {
-                  const int Ho = p.H / 2, Wo = p.W / 2;
-                  p.y[(((size_t)T.n * p.Co + o) * Ho + (row >> 1)) * Wo + (col >> 1)] = fmaxf(m, m2);
-                }
+                if (((col & 1) == 0) && in0) ybase[o * HWo + poff] = fmaxf(m, m2);
               }
             }
           }
@@ -702,6 +727,7 @@ void tc_geometry(const TcLayout& T, int W, int* ori, int* tw) {
 
 pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N, int H,
                     int W, int flags, cudaStream_t stream) {
+  if ((int64_t)M.Co * H * W >= ((int64_t)1 << 31)) return PP_ERR_UNSUPPORTED;  // 32-bit offsets within an image
   if (tc_prepare() != PP_OK) return PP_ERR_CUDA;
   TcParams p;
   p.x = x;

@@ -130,6 +130,36 @@ def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
         check_within(g, y, s, f"tensor-core kernel {(N, Ci, Co, H, W)}")
 
 
+@pytest.mark.parametrize("shape", [(12, 256, 256, 56, 56), (8, 64, 64, 128, 128)])
+def test_tensor_core_repeatable_multi_tile(pp, runner, oracle_mod, shape):
+    """Several tiles per persistent CTA, so every operand ring and both accumulator
+    buffers wrap many times.  The kernel's summation order is fixed, so repeated
+    runs must agree bit for bit (a pipeline race shows up as a run-to-run
+    difference); one run is also checked against the oracle on sampled outputs."""
+    N, Ci, Co, H, W = shape
+    rng = np.random.default_rng(Ci + W)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=1.0)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    dl = runner.DeviceLayer(L)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC)
+        xd = dev(x)
+        outs = []
+        for _ in range(5):
+            y = torch.full((N, Co, H, W), float("nan"), device="cuda")
+            dl.forward(xd, y, None, N, H, W, 0, torch.cuda.current_stream())
+            outs.append(y)
+        torch.cuda.synchronize()
+        for k in range(1, 5):
+            assert torch.equal(outs[0], outs[k]), f"run {k} differs from run 0"
+        assert pp.pp_layer_device_status(dl.handle) == 0
+        pts = sample_points(rng, N, Co, H, W, 2000)
+        yr, s = oracle_layer_points(oracle_mod, L, x, pts)
+        check_within(outs[0].cpu().numpy()[tuple(pts.T)], yr, s, f"multi-tile {shape}")
+    finally:
+        dl.close()
+
+
 def test_autotune_keeps_parity(pp, runner, oracle_mod):
     rng = np.random.default_rng(44)
     L = synth.small_random_layer(rng, 96, 64, P=8, keep=0.4)
