@@ -149,6 +149,16 @@ pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const
  *   PP_KERNEL_TC        implicit GEMM on the tensor cores over the 9 taps
  *                       (zeros where pruned), 3xTF32 for fp32 accuracy; any
  *                       pattern set; needs Ci >= 8.
+ *   PP_KERNEL_TC_FLAT   the same contraction with whole output rows flattened
+ *                       into one MMA and, for layers with few output tiles,
+ *                       the input channels split over a thread-block cluster;
+ *                       maps at most 128 pixels wide and layers with more than
+ *                       64 filters (other shapes run PP_KERNEL_TC).  A split
+ *                       launch keeps fp32 partial tiles in a workspace owned
+ *                       by the layer, allocated on first use outside stream
+ *                       capture (inside a capture without one, the launch
+ *                       runs unsplit); so calls of one layer must not run
+ *                       concurrently on different streams.
  *   PP_KERNEL_TMEM      FP32 FMA over kept taps only, accumulators in tensor
  *                       memory; ring patterns only (the centre tap plus 3
  *                       consecutive of its 8 neighbours).
@@ -160,8 +170,9 @@ pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const
 #define PP_KERNEL_TMEM 1
 #define PP_KERNEL_REGISTER 2
 #define PP_KERNEL_TC 3
+#define PP_KERNEL_TC_FLAT 4
 pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
-/* The kernel that pp_conv_forward will run (PP_KERNEL_TC, _TMEM or _REGISTER). */
+/* The kernel that pp_conv_forward will run (one of the PP_KERNEL_ values above, not _AUTO). */
 pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
 /* Time every kernel that can run this layer on zero-filled scratch tensors of
  * the given shape and flags (a few launches each, on stream, synchronous) and

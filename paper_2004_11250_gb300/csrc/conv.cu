@@ -553,13 +553,18 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   if ((flags & PP_ADD_SKIP) && !skip) return PP_ERR_INVALID_ARG;
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   if (((uintptr_t)y & 15) || ((uintptr_t)x & 3)) return PP_ERR_INVALID_ARG;
-  if (L->kernel == PP_KERNEL_TMEM || L->kernel == PP_KERNEL_TC) {
+  if (L->kernel == PP_KERNEL_TMEM || L->kernel == PP_KERNEL_TC || L->kernel == PP_KERNEL_TC_FLAT) {
     ppc::LayerMeta M;
     M.Co = L->Co;
     M.Ci = L->Ci;
     M.perm = L->perm;
     M.bias = L->has_bias ? L->bias : nullptr;
-    if (L->kernel == PP_KERNEL_TC) {
+    if (L->kernel == PP_KERNEL_TC_FLAT) {
+      const pp_status st = ppc::tcf_launch(L->tc, M, x, y, skip, N, H, W, flags, stream);
+      if (st != PP_ERR_UNSUPPORTED) return st;
+      // maps wider than the flat kernel's tiles run the row-tiled tensor-core kernel
+    }
+    if (L->kernel == PP_KERNEL_TC || L->kernel == PP_KERNEL_TC_FLAT) {
       const pp_status st = ppc::tc_launch(L->tc, M, x, y, skip, N, H, W, flags, stream);
       if (st != PP_ERR_UNSUPPORTED) return st;
       // shapes beyond the tensor-core kernel's 32-bit offsets run on an FMA kernel
@@ -677,7 +682,8 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
   const double nk = (double)pk->kidx.size();
   const double tc_cycles = 27.0 * (double)((pk->Co + 127) / 128 * 128) * (double)((pk->Ci + 7) / 8 * 8) / 1800.0;
   const double fma_cycles = 4.0 * nk / 32.0;
-  L->auto_kernel = (L->tc_ok && tc_cycles < fma_cycles) ? PP_KERNEL_TC : (L->tm_ok ? PP_KERNEL_TMEM : PP_KERNEL_REGISTER);
+  L->auto_kernel = (L->tc_ok && tc_cycles < fma_cycles) ? (L->tc.FB == 128 ? PP_KERNEL_TC_FLAT : PP_KERNEL_TC)
+                                                         : (L->tm_ok ? PP_KERNEL_TMEM : PP_KERNEL_REGISTER);
   L->kernel = L->auto_kernel;
   *out = L;
   return PP_OK;
@@ -693,6 +699,10 @@ extern "C" pp_status pp_layer_set_kernel(pp_layer* L, int kernel) {
       return PP_OK;
     case PP_KERNEL_TC:
       if (!L->tc_ok) return PP_ERR_UNSUPPORTED;
+      L->kernel = kernel;
+      return PP_OK;
+    case PP_KERNEL_TC_FLAT:
+      if (!L->tc_ok || L->tc.FB != 128) return PP_ERR_UNSUPPORTED;
       L->kernel = kernel;
       return PP_OK;
     case PP_KERNEL_REGISTER: L->kernel = kernel; return PP_OK;
@@ -713,6 +723,7 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
   cudaStream_t stream = (cudaStream_t)stream_;
   std::vector<int> cand;
   if (L->tc_ok) cand.push_back(PP_KERNEL_TC);
+  if (L->tc_ok && L->tc.FB == 128) cand.push_back(PP_KERNEL_TC_FLAT);
   if (L->tm_ok) cand.push_back(PP_KERNEL_TMEM);
   if (cand.empty()) cand.push_back(PP_KERNEL_REGISTER);
   if (cand.size() == 1) {
@@ -794,7 +805,7 @@ extern "C" void pp_layer_destroy(pp_layer* L) {
   if (!L) return;
   if (L->dmem) cudaFree(L->dmem);
   if (L->tm.dmem) cudaFree(L->tm.dmem);
-  if (L->tc.dmem) cudaFree(L->tc.dmem);
+  ppc::tc_free(&L->tc);
   delete L;
 }
 

@@ -47,8 +47,11 @@
 #include <vector>
 
 #include "internal.h"
+#include "tc_ptx.cuh"
 
 namespace {
+
+using namespace ppc_ptx;
 
 constexpr int KC = 8;              // input channels per chunk (MMA K for tf32)
 constexpr int NTAP = 9;
@@ -80,77 +83,6 @@ struct TcParams {
   int flags;
   int use_tma;  // input tiles by tensor-map copy (W % 4 == 0, aligned x), else per-thread loads
 };
-
-__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-// Shared-memory matrix descriptor, K-major, no swizzle: core matrices of 8 rows
-// x 16 bytes; lbo = byte distance between the two K halves, sbo = 128 between
-// groups of 8 rows; bit 46 = descriptor version of this architecture.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo) {
-  uint64_t d = (uint64_t)((addr >> 4) & 0x3FFF);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
-  d |= (uint64_t)(128 >> 4) << 32;
-  d |= (uint64_t)1 << 46;
-  return d;
-}
-
-// Instruction descriptor: D f32, A and B tf32, both K-major, shape M x N.
-__host__ __device__ constexpr uint32_t idesc_tf32(int m, int n) {
-  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t a, int count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count));
-}
-__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
-  uint32_t ok;
-  asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
-               : "=r"(ok)
-               : "r"(a), "r"(parity)
-               : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t a) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
-}
-// Add an expected transaction count without arriving.
-__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
-  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t a, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
-}
-// Named barrier over the loader warps only.  Every loader thread reaches each
-// use of it: loop exits are decided together with loader_any.
-__device__ __forceinline__ void loader_sync() { asm volatile("bar.sync 1, %0;" ::"n"(NLOAD) : "memory"); }
-// OR of v over the loader threads (a barrier too), so all of them take the same branch.
-__device__ __forceinline__ bool loader_any(bool v) {
-  uint32_t r;
-  asm volatile("{ .reg .pred p, q; setp.ne.u32 p, %1, 0; bar.red.or.pred q, 1, %2, p; selp.u32 %0, 1, 0, q; }"
-               : "=r"(r)
-               : "r"((uint32_t)v), "n"(NLOAD)
-               : "memory");
-  return r != 0;
-}
-
-__device__ __forceinline__ void tm_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tm_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tm_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void tm_ld16(uint32_t ta, float (&v)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-      : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]), "=f"(v[7]), "=f"(v[8]),
-        "=f"(v[9]), "=f"(v[10]), "=f"(v[11]), "=f"(v[12]), "=f"(v[13]), "=f"(v[14]), "=f"(v[15])
-      : "r"(ta));
-}
-__device__ __forceinline__ void mma_tf32(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc) {
-  asm volatile(
-      "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p; }" ::"r"(d),
-      "l"(a), "l"(b), "r"(id), "r"(acc));
-}
-__device__ __forceinline__ void mma_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
-}
 
 // Geometry of one instantiation.  TW pixels per output row segment, FB filters
 // per block, R row segments per tile (one accumulator column range each).
@@ -273,7 +205,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
       for (int c = 0; c < p.nch; ++c, ++g) {
         const int s = g & 1, use = g >> 1;
-        if (loader_any(use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1)))) {
+        if (group_any<NLOAD>(use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1)))) {
           stop = true;
           break;
         }
@@ -296,7 +228,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         }
         const int ch0 = c * KC;
         if (p.use_tma) {
-          if (loader_any(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
+          if (group_any<NLOAD>(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
             stop = true;
             break;
           }
@@ -317,7 +249,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           // each thread orders its generic-proxy reads of the slot before that
           // copy with a proxy fence, then the loader barrier lets thread 0 issue it.
           if (G::SEP) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          loader_sync();  // every raw value is in registers before its slot is reused
+          group_sync<NLOAD>();  // every raw value is in registers before its slot is reused
           if (G::SEP && tid == 0 && raw_issued < nall && raw_issued == g + 2) {
             issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued & 1) * G::RAW);
             ++raw_issued;
@@ -707,6 +639,11 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
     cudaFree(d);
     return PP_ERR_CUDA;
   }
+  T->scratch = new (std::nothrow) TcScratch();
+  if (!T->scratch) {
+    cudaFree(d);
+    return PP_ERR_OOM;
+  }
   T->dmem = d;
   T->dbytes = total + 256;
   T->a = static_cast<const unsigned char*>(d);
@@ -764,6 +701,16 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
     return PP_ERR_CUDA;
   }
   return PP_OK;
+}
+
+void tc_free(TcLayout* T) {
+  if (T->dmem) cudaFree(T->dmem);
+  T->dmem = nullptr;
+  if (T->scratch) {
+    if (T->scratch->p) cudaFree(T->scratch->p);
+    delete T->scratch;
+    T->scratch = nullptr;
+  }
 }
 
 pp_status tc_status(const TcLayout& T, int* device_error) {

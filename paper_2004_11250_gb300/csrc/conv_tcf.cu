@@ -1,0 +1,756 @@
+// Pattern-pruned 3x3 convolution on the tensor cores, "flat" variant for maps
+// at most 128 pixels wide, with the input-channel loop optionally split over a
+// thread-block cluster.
+//
+// The layer is the same dense contraction as in conv_tc.cu (pruned taps and
+// kernels written as zeros, Section 2; 3xTF32 split for fp32 accuracy), with a
+// different mapping of the output tile onto one MMA:
+//   * M = 128 consecutive reordered filters (TMEM lanes);
+//   * N = the pixels of R whole output rows, flattened.  The input tile for a
+//     chunk of 8 channels is staged as R + 2 rows of BCOLS >= W + 2 pixels (zero
+//     halo, BCOLS a multiple of 8), one 16-byte K-major row per pixel.  Output
+//     pixel (r, c) of the tile is MMA column j = r * BCOLS + c, and its tap
+//     (dy, dx) reads staged pixel j + dy * BCOLS + dx, so a tap is the whole
+//     staged tile with the operand start moved by dy * BCOLS + dx pixels: one
+//     MMA of N = R * BCOLS (rounded up to 16, at most 256) per tap and pass.
+//     Columns c >= W of each row are computed and discarded.
+// Against one MMA per output row (N = tile width) this makes narrow maps
+// (14 ... 128 pixels) run full-width MMAs and halves the shared-memory operand
+// traffic per multiply-add.
+//
+// Split: when the layer has fewer output tiles than SMs, S CTAs of a cluster
+// share a tile, each summing a contiguous range of the channel chunks.  Each
+// writes its fp32 partial tile to a workspace in global memory (it stays in
+// L2), the cluster barrier orders those writes before the reads, and each CTA
+// then finishes 1/S of the tile's filters: bulk copies bring the S partials of
+// those filters into shared memory, where they are added in rank order
+// (deterministic), then bias, skip, ReLU, pool, and y is stored.
+//
+// Roles (17 warps, one CTA per SM): warps 0-7 stage the operands, warp 8
+// allocates TMEM and one of its threads issues the MMAs, warps 9-16 are the
+// epilogue (two per TMEM lane quadrant).  Without a split the CTA is persistent
+// over tiles with two TMEM accumulator buffers, so a tile's epilogue overlaps
+// the next tile's MMAs.  Every mbarrier wait is bounded; a timeout sets the
+// layer's device status word and the CTA skips the rest of its work (every
+// thread still reaches the cluster barrier).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+
+#include "internal.h"
+#include "tc_ptx.cuh"
+
+namespace {
+
+using namespace ppc_ptx;
+
+constexpr int KC = 8;                 // input channels per chunk (MMA K for tf32)
+constexpr int NTAP = 9;
+constexpr int FB = 128;               // filters per block (MMA M)
+constexpr int NMAX = 256;             // TMEM columns of one accumulator buffer
+constexpr int NLOAD = 256;            // loader threads (warps 0-7)
+constexpr int MMA_WARP = 8;
+constexpr int EPI_WARP0 = 9;          // warps 9-16
+constexpr int NEPI = 256;
+constexpr int NTHREADS = 544;
+constexpr int WMAX = 128;             // widest map handled
+constexpr int W_TILE = FB * KC * 4;   // one tap, hi or lo: 128 x 8 fp32
+constexpr int W_BYTES = NTAP * 2 * W_TILE;
+constexpr int PIX_MAX = 544;          // staged pixels per K half, padding included
+constexpr int IN_HALF_MAX = PIX_MAX * 16;
+constexpr int IN_MAX = 2 * IN_HALF_MAX;  // hi (or lo) operand of one chunk
+constexpr int LO_MAX = IN_MAX;        // lo operand; the raw tensor-map box lands here first
+constexpr int STAGE = W_BYTES + IN_MAX + LO_MAX;
+constexpr int SMEM_ALLOC = 2 * STAGE + 1024;
+constexpr int ITEMS_MAX = (2 * PIX_MAX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
+constexpr int PF_AHEAD = 6;           // chunks whose operands are prefetched into L2 ahead of use
+constexpr long WAIT_LIMIT = 1L << 22;
+constexpr int MAX_SPLIT = 16;
+static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
+static_assert(STAGE % 128 == 0 && (W_BYTES + IN_MAX) % 128 == 0, "stage alignment");
+
+struct FlatParams {
+  const float* x;
+  float* y;
+  const float* skip;
+  const unsigned char* wt;  // [nfb][nch][9][2][128 x 8] canonical tiles
+  const int* perm;
+  const float* bias;
+  int* status;
+  float* ws;                // split partials [grid][128][ncols]
+  int N, Ci, Co, H, W;
+  int nch, nfb, flags, use_tma;
+  int bcols, R, ncols, npix, npixa, raw_w, raw_bytes;
+  int tiles_y, ntiles, split;
+  uint32_t idesc;
+};
+
+struct Tile {
+  int n, r0, fb;
+};
+__device__ __forceinline__ Tile tile_of(const FlatParams& p, int t) {
+  Tile T;
+  T.fb = t % p.nfb;
+  t /= p.nfb;
+  T.r0 = (t % p.tiles_y) * p.R;
+  T.n = t / p.tiles_y;
+  return T;
+}
+
+template <bool SPLIT>
+__global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t full[2], wfull[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar, red_bar;
+  __shared__ uint32_t tmem_s;
+  __shared__ volatile int abort_s;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  auto wait = [&](uint64_t* bar, uint32_t parity) -> bool {
+    const uint32_t a = su32(bar);
+    for (long i = 0; i < WAIT_LIMIT; ++i) {
+      if (mbar_try(a, parity)) return true;
+      if ((i & 255) == 255 && abort_s) return false;
+    }
+    abort_s = 1;
+    atomicExch(p.status, 1);
+    return false;
+  };
+
+  if (tid == 0) {
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(su32(&full[s]), NLOAD);
+      mbar_init(su32(&wfull[s]), 1);
+      mbar_init(su32(&raw_full[s]), 1);
+      mbar_init(su32(&empty[s]), 1);
+      mbar_init(su32(&acc_full[s]), 1);
+      mbar_init(su32(&acc_empty[s]), NEPI);
+    }
+    mbar_init(su32(&done_bar), 1);
+    mbar_init(su32(&red_bar), 1);
+    abort_s = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == MMA_WARP) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&tmem_s)),
+                 "n"(2 * NMAX));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tm_fence_before();
+  __syncthreads();
+  tm_fence_after();
+  const uint32_t tmem = tmem_s;
+
+  // This CTA's tiles and channel-chunk range.
+  int nmine, c_beg, c_end;
+  if (SPLIT) {
+    const int rank = (int)blockIdx.x % p.split;
+    nmine = 1;
+    c_beg = rank * p.nch / p.split;
+    c_end = (rank + 1) * p.nch / p.split;
+  } else {
+    nmine = p.ntiles > (int)blockIdx.x ? (p.ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    c_beg = 0;
+    c_end = p.nch;
+  }
+  auto tile_index = [&](int i) -> int {
+    return SPLIT ? (int)blockIdx.x / p.split : (int)blockIdx.x + i * (int)gridDim.x;
+  };
+  const int brows = p.R + 2;
+
+  if (warp < MMA_WARP) {
+    // ------------------------------------------------------------ loaders
+    // Chunk sequence g = 0 .. nall-1 of this CTA (tiles in order, each over the
+    // CTA's chunk range).  Thread 0 keeps the weights (and input boxes) of the
+    // next PF_AHEAD chunks on their way into L2, so the copies into shared
+    // memory, which wait for a free stage, find them there.
+    const int nchm = c_end - c_beg;
+    const int nall = nmine * nchm;
+    auto prefetch = [&](int gg) {  // thread 0 only
+      const int i = gg / nchm, c = c_beg + gg % nchm;
+      const Tile T = tile_of(p, tile_index(i));
+      const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(W_BYTES) : "memory");
+      if (p.use_tma)
+        asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                         reinterpret_cast<uint64_t>(&xmap)),
+                     "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n)
+                     : "memory");
+    };
+    if (tid == 0)
+      for (int gg = 0; gg < PF_AHEAD && gg < nall; ++gg) prefetch(gg);
+    int g = 0, w_issued = 0, raw_issued = 0;
+    bool stop = false;  // identical in every loader thread (decided by group_any)
+    for (int i = 0; i < nmine && !stop; ++i) {
+      const Tile T = tile_of(p, tile_index(i));
+      const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
+      for (int c = c_beg; c < c_end; ++c, ++g) {
+        const int s = g & 1, use = g >> 1;
+        // Without a tensor map the chunk's input values are fetched into
+        // registers first: that needs no free stage, so it overlaps the wait.
+        float v[ITEMS_MAX][4];
+        if (!p.use_tma) {
+#pragma unroll
+          for (int b = 0; b < ITEMS_MAX; ++b) {
+            const int it = b * NLOAD + tid;
+            const int kh = it >= p.npix ? 1 : 0;
+            const int pix = it - kh * p.npix;
+            const int br = pix / p.bcols, bc = pix - br * p.bcols;
+            const int r = T.r0 - 1 + br, cc = bc - 1;
+            const bool inside = it < 2 * p.npix && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int ch = c * KC + kh * 4 + k;
+              v[b][k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
+            }
+          }
+        }
+        if (group_any<NLOAD>(use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1)))) {
+          stop = true;
+          break;
+        }
+        unsigned char* st = smem + s * STAGE;
+        float4* hi = reinterpret_cast<float4*>(st + W_BYTES);
+        float4* lo = reinterpret_cast<float4*>(st + W_BYTES + IN_MAX);
+        if (tid == 0) {
+          const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
+          mbar_arrive_expect_tx(su32(&wfull[s]), W_BYTES);
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(su32(st)),
+              "l"(src), "r"(W_BYTES), "r"(su32(&wfull[s]))
+              : "memory");
+          ++w_issued;
+          if (p.use_tma) {
+            // box [8 channels][rows r0-1 ..][columns -4 ..]; zero fill outside the
+            // image is the convolution's padding
+            mbar_arrive_expect_tx(su32(&raw_full[s]), (uint32_t)p.raw_bytes);
+            asm volatile(
+                "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+                "%4, %5}], [%6];" ::"r"(su32(lo)),
+                "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
+                "r"(su32(&raw_full[s]))
+                : "memory");
+            ++raw_issued;
+          }
+          if (g + PF_AHEAD < nall) prefetch(g + PF_AHEAD);
+        }
+        if (p.use_tma) {
+          if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
+            stop = true;
+            break;
+          }
+          const float* raw = reinterpret_cast<const float*>(lo);
+#pragma unroll
+          for (int b = 0; b < ITEMS_MAX; ++b) {
+            const int it = b * NLOAD + tid;
+            const int kh = it >= p.npix ? 1 : 0;
+            const int pix = it - kh * p.npix;
+            const int br = pix / p.bcols, bc = pix - br * p.bcols;
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              v[b][k] = it < 2 * p.npix ? raw[((kh * 4 + k) * brows + br) * p.raw_w + bc + 3] : 0.f;
+          }
+          group_sync<NLOAD>();  // the whole box is in registers before lo is overwritten
+        }
+#pragma unroll
+        for (int b = 0; b < ITEMS_MAX; ++b) {
+          const int it = b * NLOAD + tid;
+          if (it < 2 * p.npix) {
+            const int kh = it >= p.npix ? 1 : 0;
+            const int dst = kh * p.npixa + it - kh * p.npix;
+            float4 h;
+            h.x = tf32_hi(v[b][0]);
+            h.y = tf32_hi(v[b][1]);
+            h.z = tf32_hi(v[b][2]);
+            h.w = tf32_hi(v[b][3]);
+            hi[dst] = h;
+            lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+          }
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        mbar_arrive(su32(&full[s]));
+      }
+    }
+    if (tid == 0) {
+      // No copy may still be writing shared memory when the CTA exits: wait
+      // (bounded) for the last copies issued into each stage.
+      for (int gg = raw_issued > 2 ? raw_issued - 2 : 0; gg < raw_issued; ++gg)
+        for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&raw_full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+        }
+      for (int gg = w_issued > 2 ? w_issued - 2 : 0; gg < w_issued; ++gg)
+        for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&wfull[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+        }
+    }
+    __syncwarp();
+  } else if (warp == MMA_WARP) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int g = 0;
+      for (int i = 0; i < nmine && !abort_s; ++i) {
+        const int b = i & 1, ub = i >> 1;
+        if (ub > 0 && !wait(&acc_empty[b], (uint32_t)((ub - 1) & 1))) break;
+        tm_fence_after();
+        const uint32_t d = tmem + (uint32_t)(b * NMAX);
+        bool okc = true;
+        for (int c = c_beg; c < c_end; ++c, ++g) {
+          const int s = g & 1, use = g >> 1;
+          if (!wait(&full[s], (uint32_t)(use & 1)) || !wait(&wfull[s], (uint32_t)(use & 1))) {
+            okc = false;
+            break;
+          }
+          tm_fence_after();
+          const unsigned char* st = smem + s * STAGE;
+          // descriptors hold address / 16 in their low 14 bits (operands lie below
+          // 256 KB), so moving an operand by k pixels of 16 bytes adds k
+          const uint64_t w0 = smem_desc(su32(st), FB * 16);
+          const uint64_t xh0 = smem_desc(su32(st + W_BYTES), (uint32_t)p.npixa * 16);
+          const uint64_t xl0 = smem_desc(su32(st + W_BYTES + IN_MAX), (uint32_t)p.npixa * 16);
+          const uint32_t acc0 = c == c_beg ? 0u : 1u;  // the range's first chunk overwrites the accumulators
+#pragma unroll
+          for (int t = 0; t < NTAP; ++t) {
+            const uint64_t off = (uint64_t)((t / 3) * p.bcols + t % 3);
+            const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * W_TILE / 16);
+            const uint64_t wlo = w0 + (uint64_t)((t * 2 + 1) * W_TILE / 16);
+            mma_tf32(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+            mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
+            mma_tf32(d, whi, xl0 + off, p.idesc, 1u);
+          }
+          mma_commit(su32(&empty[s]));
+        }
+        if (!okc) break;
+        mma_commit(su32(&acc_full[b]));
+      }
+      // every MMA issued by this thread is complete before TMEM is released
+      mma_commit(su32(&done_bar));
+      wait(&done_bar, 0u);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;                     // TMEM lane quadrant of this warp
+    const int half = (warp - EPI_WARP0) >> 2;   // the two warps of a quadrant share the work
+    const bool pool = p.flags & PP_POOL2;
+    const bool relu = p.flags & PP_RELU;
+    const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
+    for (int i = 0; i < nmine; ++i) {
+      const int b = i & 1, ub = i >> 1;
+      // the whole warp leaves together: its TMEM loads are warp-collective
+      if (!__all_sync(0xffffffffu, wait(&acc_full[b], (uint32_t)(ub & 1)))) break;
+      tm_fence_after();
+      const Tile T = tile_of(p, tile_index(i));
+      const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NMAX);
+      const int m = 32 * q + lane;  // filter within the block = TMEM lane
+      if (SPLIT) {
+        // this CTA's partial tile, row m of [128][ncols] at its grid index
+        float* wrow = p.ws + ((size_t)blockIdx.x * FB + m) * p.ncols;
+        for (int cb = half * 8; cb < p.ncols; cb += 16) {
+          float a[8];
+          tm_ld8(lanebase + (uint32_t)cb, a);
+          tm_wait_ld();
+          *reinterpret_cast<float4*>(wrow + cb) = make_float4(a[0], a[1], a[2], a[3]);
+          *reinterpret_cast<float4*>(wrow + cb + 4) = make_float4(a[4], a[5], a[6], a[7]);
+        }
+        // the partial is read back by bulk copies (async proxy) in other CTAs
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+      } else {
+        const int jr = T.fb * FB + m;
+        const bool valid = jr < p.Co;
+        const int o = valid ? __ldg(p.perm + jr) : 0;
+        const float bs = (valid && p.bias) ? __ldg(p.bias + jr) : 0.f;
+        const size_t plane = (size_t)T.n * p.Co + o;
+        const bool vec = (p.W & 3) == 0;
+        if (!pool) {
+          for (int rr = half; rr < p.R; rr += 2) {
+            const int row = T.r0 + rr;
+            if (row >= p.H) break;
+            float* yr = p.y + (plane * p.H + row) * p.W;
+            const float* sr = skip ? skip + (plane * p.H + row) * p.W : nullptr;
+            for (int cb = 0; cb < p.W; cb += 8) {
+              float a[8];
+              tm_ld8(lanebase + (uint32_t)(rr * p.bcols + cb), a);
+              tm_wait_ld();
+              if (valid) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                  a[k] += bs;
+                  if (sr && cb + k < p.W) a[k] += __ldg(sr + cb + k);
+                  if (relu) a[k] = fmaxf(a[k], 0.f);
+                }
+                if (vec && cb + 8 <= p.W) {
+                  *reinterpret_cast<float4*>(yr + cb) = make_float4(a[0], a[1], a[2], a[3]);
+                  *reinterpret_cast<float4*>(yr + cb + 4) = make_float4(a[4], a[5], a[6], a[7]);
+                } else {
+#pragma unroll
+                  for (int k = 0; k < 8; ++k)
+                    if (cb + k < p.W) yr[cb + k] = a[k];
+                }
+              }
+            }
+          }
+        } else {
+          const int Ho = p.H / 2, Wo = p.W / 2;
+          for (int rr = 2 * half; rr < p.R; rr += 4) {
+            const int row = T.r0 + rr;
+            if (row >= p.H) break;
+            float* yr = p.y + (plane * Ho + row / 2) * Wo;
+            const float* s0 = skip ? skip + (plane * p.H + row) * p.W : nullptr;
+            for (int cb = 0; cb < p.W; cb += 8) {
+              float a[8], bb[8];
+              tm_ld8(lanebase + (uint32_t)(rr * p.bcols + cb), a);
+              tm_ld8(lanebase + (uint32_t)((rr + 1) * p.bcols + cb), bb);
+              tm_wait_ld();
+              if (valid) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                  a[k] += bs;
+                  bb[k] += bs;
+                  if (s0 && cb + k < p.W) {
+                    a[k] += __ldg(s0 + cb + k);
+                    bb[k] += __ldg(s0 + p.W + cb + k);
+                  }
+                  if (relu) {
+                    a[k] = fmaxf(a[k], 0.f);
+                    bb[k] = fmaxf(bb[k], 0.f);
+                  }
+                }
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                  if (cb + 2 * k < p.W)
+                    yr[cb / 2 + k] = fmaxf(fmaxf(a[2 * k], a[2 * k + 1]), fmaxf(bb[2 * k], bb[2 * k + 1]));
+              }
+            }
+          }
+        }
+      }
+      tm_fence_before();
+      mbar_arrive(su32(&acc_empty[b]));
+    }
+  }
+
+  if (SPLIT) {
+    // Every thread of every CTA of the cluster arrives, also after an early
+    // stop, so the barrier always completes.  Release / acquire at cluster
+    // scope (with proxy fences on both sides, as the partials are written by
+    // plain stores and read by bulk copies) orders the partial tiles written
+    // above before the copies below.
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+    // This CTA finishes filters [m0, m1) of the tile: the S partials of those
+    // rows (contiguous in the workspace) come into shared memory, freed by the
+    // main loop, by one bulk copy each, and are added in rank order.
+    const int tile = (int)blockIdx.x / p.split, rank = (int)blockIdx.x % p.split;
+    const int m0 = rank * FB / p.split, m1 = (rank + 1) * FB / p.split, nm = m1 - m0;
+    const uint32_t slice = (uint32_t)(nm * p.ncols * 4);
+    bool issued = false;  // thread 0: the copies below were issued
+    if (tid == 0 && !abort_s) {
+      issued = true;
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      mbar_arrive_expect_tx(su32(&red_bar), slice * (uint32_t)p.split);
+      for (int s = 0; s < p.split; ++s) {
+        const float* src = p.ws + (((size_t)tile * p.split + s) * FB + m0) * p.ncols;
+        asm volatile(
+            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                su32(smem + (size_t)s * slice)),
+            "l"(src), "r"(slice), "r"(su32(&red_bar))
+            : "memory");
+      }
+    }
+    // the whole warp takes one branch (every lane runs the vote)
+    if (warp >= EPI_WARP0 && __all_sync(0xffffffffu, !abort_s && wait(&red_bar, 0u))) {
+      const int e = tid - EPI_WARP0 * 32;
+      const Tile T = tile_of(p, tile);
+      const bool pool = p.flags & PP_POOL2;
+      const bool relu = p.flags & PP_RELU;
+      const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
+      const float* buf = reinterpret_cast<const float*>(smem);  // [S][nm][ncols]
+      const int sl = nm * p.ncols;
+      const int Ro = pool ? p.R / 2 : p.R, Wo = pool ? p.W / 2 : p.W;
+      const int total = nm * Ro * Wo;
+      for (int idx = e; idx < total; idx += NEPI) {
+        const int cx = idx % Wo;
+        const int t2 = idx / Wo;
+        const int ro = t2 % Ro, ml = t2 / Ro;
+        const int jr = T.fb * FB + m0 + ml;
+        if (jr >= p.Co) continue;
+        const int o = __ldg(p.perm + jr);
+        const float bs = p.bias ? __ldg(p.bias + jr) : 0.f;
+        const size_t plane = (size_t)T.n * p.Co + o;
+        const float* src = buf + ml * p.ncols;
+        if (!pool) {
+          const int row = T.r0 + ro;
+          if (row >= p.H) continue;
+          const int col = ro * p.bcols + cx;
+          float v = 0.f;
+          for (int s = 0; s < p.split; ++s) v += src[s * sl + col];
+          v += bs;
+          const size_t yi = (plane * p.H + row) * p.W + cx;
+          if (skip) v += __ldg(skip + yi);
+          if (relu) v = fmaxf(v, 0.f);
+          p.y[yi] = v;
+        } else {
+          const int rr = 2 * ro, row = T.r0 + rr;
+          if (row >= p.H) continue;
+          float mx = 0.f;
+#pragma unroll
+          for (int d = 0; d < 4; ++d) {
+            const int dr = d >> 1, dc = d & 1;
+            const int col = (rr + dr) * p.bcols + 2 * cx + dc;
+            float v = 0.f;
+            for (int s = 0; s < p.split; ++s) v += src[s * sl + col];
+            v += bs;
+            if (skip) v += __ldg(skip + (plane * p.H + row + dr) * p.W + 2 * cx + dc);
+            if (relu) v = fmaxf(v, 0.f);
+            mx = d == 0 ? v : fmaxf(mx, v);
+          }
+          p.y[(plane * (p.H / 2) + row / 2) * (p.W / 2) + cx] = mx;
+        }
+      }
+    }
+    if (issued) {
+      // the copies have landed before the CTA exits, also if the wait above gave up
+      for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&red_bar), 0u); ++k) {
+      }
+    }
+  }
+
+  tm_fence_before();
+  __syncthreads();
+  tm_fence_after();
+  if (warp == MMA_WARP)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(2 * NMAX));
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+struct DeviceState {
+  bool ready = false;
+  int sms = 0;
+  int max_clusters[MAX_SPLIT + 1] = {};  // co-resident clusters of each size (0: size unusable)
+  EncodeTiledFn encode = nullptr;
+};
+DeviceState g_dev[64];
+
+DeviceState* prepare() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  DeviceState& D = g_dev[dev];
+  if (D.ready) return &D;
+  if (cudaDeviceGetAttribute(&D.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return nullptr;
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
+          cudaSuccess)
+    return nullptr;
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+    cudaGetLastError();  // then only portable sizes (up to 8) can be used
+  for (int s = 2; s <= MAX_SPLIT; s *= 2) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = (unsigned)s;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)s);
+    cfg.blockDim = dim3(NTHREADS);
+    cfg.dynamicSmemBytes = SMEM_ALLOC;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, ppconv_tcf_kernel<true>, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      n = 0;
+    }
+    D.max_clusters[s] = n;
+  }
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    D.encode = reinterpret_cast<EncodeTiledFn>(fn);
+  else
+    cudaGetLastError();  // without the entry point every launch uses per-thread loads
+  D.ready = true;
+  return &D;
+}
+
+struct FlatGeo {
+  int bcols = 0, R = 0, ncols = 0, npix = 0, npixa = 0, raw_w = 0, raw_bytes = 0, tiles_y = 0, ntiles = 0, split = 1;
+  double cost = 1e300;
+};
+
+// Geometry of one launch: rows per tile and split, by a model of the time in
+// SM cycles: an MMA of N columns takes the longer of its multiply-adds at
+// ~1850 per cycle and its operand reads (4 KB of weights + 32 N bytes of
+// input) at 128 shared-memory bytes per cycle; a chunk also needs its 73.7 KB
+// of weights from L2 (~48 bytes per cycle) and at least ~1500 cycles of
+// staging latency with two stages; a start-up and pipeline fill of ~5000
+// cycles; the split's partial-tile round trip through L2 at ~64 bytes per
+// cycle; and clusters beyond those co-resident on the GPU run in later waves.
+bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
+                   FlatGeo* out) {
+  if (W < 1 || W > WMAX || H < 1) return false;
+  const int bcols = (W + 2 + 7) / 8 * 8;
+  const int rmax = NMAX / bcols;
+  if (rmax < 1 || (pool && rmax < 2)) return false;
+  FlatGeo best;
+  for (int r0 = rmax; r0 >= 1; r0 = r0 / 2) {
+    int R = std::min(r0, H);
+    int ty = (H + R - 1) / R;
+    R = (H + ty - 1) / ty;  // balance the rows over the tiles
+    if (pool) {
+      R += R & 1;
+      if (R > rmax) R = rmax & ~1;
+      if (R < 2) break;
+    }
+    ty = (H + R - 1) / R;
+    FlatGeo G;
+    G.bcols = bcols;
+    G.R = R;
+    G.ncols = (R * bcols + 15) / 16 * 16;
+    G.npix = (R + 2) * bcols;
+    G.npixa = G.npix + 16;
+    G.raw_w = bcols + 4;
+    G.raw_bytes = KC * (R + 2) * G.raw_w * 4;
+    G.tiles_y = ty;
+    const int64_t nt = (int64_t)ty * nfb * N;
+    if (G.npixa > PIX_MAX || G.raw_bytes > LO_MAX || G.ncols > NMAX || nt > INT32_MAX / MAX_SPLIT) continue;
+    G.ntiles = (int)nt;
+    const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
+    const double per_chunk = std::max(std::max(mma, W_BYTES / 48.0), 1500.0);
+    for (int s = 1; s <= MAX_SPLIT; s *= 2) {
+      if (s > 1 && (!allow_split || s > nch || D.max_clusters[s] <= 0 || (int64_t)G.ntiles * s > D.sms)) continue;
+      double cost;
+      if (s == 1) {
+        const double waves = std::ceil((double)G.ntiles / D.sms);
+        cost = waves * nch * per_chunk + 5000.0;
+      } else {
+        // clusters beyond those that fit on the GPU at once run in a later wave
+        const double waves = std::ceil((double)G.ntiles / D.max_clusters[s]);
+        cost = waves * (std::ceil((double)nch / s) * per_chunk + 5000.0 + 16.0 * G.ncols);
+      }
+      if (cost < best.cost) {
+        best = G;
+        best.split = s;
+        best.cost = cost;
+      }
+    }
+    if (r0 == 1) break;
+  }
+  if (best.R == 0) return false;
+  *out = best;
+  return true;
+}
+
+}  // namespace
+
+namespace ppc {
+
+pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N, int H,
+                     int W, int flags, cudaStream_t stream) {
+  if (T.FB != FB || !T.scratch) return PP_ERR_UNSUPPORTED;
+  DeviceState* D = prepare();
+  if (!D) return PP_ERR_CUDA;
+  const bool pool = flags & PP_POOL2;
+  FlatGeo G;
+  if (!flat_geometry(N, H, W, T.nch, T.nfb, pool, true, *D, &G)) return PP_ERR_UNSUPPORTED;
+  if (G.split > 1) {
+    const size_t need = (size_t)G.ntiles * G.split * FB * G.ncols * sizeof(float);
+    if (T.scratch->bytes < need) {
+      // Grow the layer's split workspace, but never inside a stream capture:
+      // there the launch runs unsplit instead.
+      cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+      const bool capturing = cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone;
+      cudaGetLastError();
+      bool ok = false;
+      if (!capturing) {
+        if (T.scratch->p) cudaFree(T.scratch->p);
+        T.scratch->p = nullptr;
+        T.scratch->bytes = 0;
+        void* d = nullptr;
+        if (cudaMalloc(&d, need) == cudaSuccess) {
+          T.scratch->p = static_cast<float*>(d);
+          T.scratch->bytes = need;
+          ok = true;
+        } else {
+          cudaGetLastError();
+        }
+      }
+      if (!ok && !flat_geometry(N, H, W, T.nch, T.nfb, pool, false, *D, &G)) return PP_ERR_UNSUPPORTED;
+    }
+  }
+  FlatParams p;
+  p.x = x;
+  p.y = y;
+  p.skip = (flags & PP_ADD_SKIP) ? skip : nullptr;
+  p.wt = T.a;
+  p.perm = M.perm;
+  p.bias = M.bias;
+  p.status = T.status;
+  p.ws = G.split > 1 ? T.scratch->p : nullptr;
+  p.N = N;
+  p.Ci = M.Ci;
+  p.Co = M.Co;
+  p.H = H;
+  p.W = W;
+  p.nch = T.nch;
+  p.nfb = T.nfb;
+  p.flags = flags;
+  p.bcols = G.bcols;
+  p.R = G.R;
+  p.ncols = G.ncols;
+  p.npix = G.npix;
+  p.npixa = G.npixa;
+  p.raw_w = G.raw_w;
+  p.raw_bytes = G.raw_bytes;
+  p.tiles_y = G.tiles_y;
+  p.ntiles = G.ntiles;
+  p.split = G.split;
+  p.idesc = idesc_tf32(FB, G.ncols);
+  CUtensorMap xmap;
+  std::memset(&xmap, 0, sizeof(xmap));
+  p.use_tma = 0;
+  if ((W & 3) == 0 && (reinterpret_cast<uintptr_t>(x) & 15) == 0 && D->encode) {
+    // 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][8][R+2][BCOLS+4]
+    const cuuint64_t dims[4] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)M.Ci, (cuuint64_t)N};
+    const cuuint64_t strides[3] = {(cuuint64_t)W * 4, (cuuint64_t)W * H * 4, (cuuint64_t)W * H * M.Ci * 4};
+    const cuuint32_t box[4] = {(cuuint32_t)G.raw_w, (cuuint32_t)(G.R + 2), (cuuint32_t)KC, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    p.use_tma = D->encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(x), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+                      ? 1
+                      : 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[1];
+  cfg.blockDim = dim3(NTHREADS);
+  cfg.dynamicSmemBytes = SMEM_ALLOC;
+  cfg.stream = stream;
+  cudaError_t e;
+  if (G.split > 1) {
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = (unsigned)G.split;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3((unsigned)(G.ntiles * G.split));
+    e = cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true>, p, xmap);
+  } else {
+    cfg.gridDim = dim3((unsigned)std::min(G.ntiles, D->sms));
+    e = cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false>, p, xmap);
+  }
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return PP_ERR_CUDA;
+  }
+  return PP_OK;
+}
+
+}  // namespace ppc

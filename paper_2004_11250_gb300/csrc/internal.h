@@ -47,13 +47,22 @@ struct TmLayout {
   const uint4* blob = nullptr;
 };
 
-// Dense per-tap tf32 hi/lo weight tiles of the tensor-core kernel (conv_tc.cu).
+// Workspace of the split (cluster) launches of the flat tensor-core kernel:
+// one fp32 partial output tile per CTA.  Grown on demand outside stream capture.
+struct TcScratch {
+  float* p = nullptr;
+  size_t bytes = 0;
+};
+
+// Dense per-tap tf32 hi/lo weight tiles of the tensor-core kernels (conv_tc.cu,
+// conv_tcf.cu).
 struct TcLayout {
   int FB = 128, nfb = 0, nch = 0;
   void* dmem = nullptr;
   size_t dbytes = 0;
   const unsigned char* a = nullptr;
-  int* status = nullptr;  // device word, nonzero after a timed-out wait
+  int* status = nullptr;        // device word, nonzero after a timed-out wait
+  TcScratch* scratch = nullptr;  // owned; see tc_free
 };
 
 pp_status tc_prepare();
@@ -61,6 +70,11 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream);
 pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
                     int H, int W, int flags, cudaStream_t stream);
 pp_status tc_status(const TcLayout& T, int* device_error);
+void tc_free(TcLayout* T);
+// Flat variant (maps up to 128 pixels wide, 128-filter blocks); returns
+// PP_ERR_UNSUPPORTED for shapes it does not handle.
+pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
+                     int H, int W, int flags, cudaStream_t stream);
 
 // True when every pattern of the set is one of the ring patterns (centre plus
 // 3 consecutive neighbours); ring_of[p] receives its ring index.

@@ -37,6 +37,7 @@ PP_KERNEL_AUTO = 0
 PP_KERNEL_TMEM = 1
 PP_KERNEL_REGISTER = 2
 PP_KERNEL_TC = 3
+PP_KERNEL_TC_FLAT = 4
 
 PP_ADD_SKIP = 1
 PP_RELU = 2

@@ -130,10 +130,59 @@ def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
         check_within(g, y, s, f"tensor-core kernel {(N, Ci, Co, H, W)}")
 
 
-@pytest.mark.parametrize("shape", [(12, 256, 256, 56, 56), (8, 64, 64, 128, 128)])
-def test_tensor_core_repeatable_multi_tile(pp, runner, oracle_mod, shape):
+FLAT_CASES = [
+    # N, Ci, Co, H, W: every map width class, ragged filter blocks and channel
+    # chunks, tiles that overhang the map, split and persistent launches
+    (1, 72, 130, 14, 14),
+    (1, 136, 256, 28, 28),
+    (2, 20, 200, 18, 30),
+    (1, 64, 129, 56, 56),
+    (3, 24, 160, 12, 8),
+    (1, 16, 130, 22, 112),
+    (1, 40, 192, 10, 126),
+    (1, 48, 136, 6, 128),
+    (4, 32, 256, 20, 20),
+    (1, 8, 136, 3, 2),
+]
+
+
+@pytest.mark.parametrize("case", FLAT_CASES)
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+def test_tensor_core_flat_kernel(pp, runner, oracle_mod, case, flags):
+    """The flat tensor-core kernel (whole rows per MMA, cluster split for few tiles) against the oracle."""
+    N, Ci, Co, H, W = case
+    if flags == "pool_relu" and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(11 * sum(case) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.45, ring=sum(case) % 2 == 0)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=pp.PP_KERNEL_TC_FLAT)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
+    check_within(g, y, s, f"flat tensor-core kernel {case} {flags}")
+
+
+@pytest.mark.parametrize("shape", [(1, 136, 130, 28, 28), (6, 40, 200, 14, 14)])
+def test_tensor_core_flat_integer_bit_exact(pp, runner, oracle_mod, shape):
+    """Integer weights and inputs: tf32 holds them exactly (lo parts are zero) and
+    every partial sum, including the split's partial tiles, is an exact fp32
+    integer, so the flat kernel equals the oracle bit for bit."""
+    N, Ci, Co, H, W = shape
+    rng = np.random.default_rng(Co + W)
+    L = synth.integer_layer(rng, Co, Ci, synth.ring8_patterns(), 0.5)
+    x = rng.integers(-8, 9, (N, Ci, H, W)).astype(np.float32)
+    g = run_layer(pp, runner, L, x, None, True, False, kernel=pp.PP_KERNEL_TC_FLAT)
+    y, _ = oracle_layer_full(oracle_mod, L, x, None, True, False)
+    assert (g.astype(np.float64) == y).all()
+
+
+@pytest.mark.parametrize("shape,kernel", [((12, 256, 256, 56, 56), "TC"), ((8, 64, 64, 128, 128), "TC"),
+                                          ((12, 256, 256, 56, 56), "TC_FLAT"), ((1, 512, 512, 28, 28), "TC_FLAT"),
+                                          ((1, 512, 512, 14, 14), "TC_FLAT"), ((2, 128, 128, 112, 112), "TC_FLAT")])
+def test_tensor_core_repeatable_multi_tile(pp, runner, oracle_mod, shape, kernel):
     """Several tiles per persistent CTA, so every operand ring and both accumulator
-    buffers wrap many times.  The kernel's summation order is fixed, so repeated
+    buffers wrap many times, or (flat kernel, few tiles) channel chunks split over
+    clusters.  The kernels' summation order is fixed, so repeated
     runs must agree bit for bit (a pipeline race shows up as a run-to-run
     difference); one run is also checked against the oracle on sampled outputs."""
     N, Ci, Co, H, W = shape
@@ -142,7 +191,7 @@ def test_tensor_core_repeatable_multi_tile(pp, runner, oracle_mod, shape):
     x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
     dl = runner.DeviceLayer(L)
     try:
-        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC)
+        pp.pp_layer_set_kernel(dl.handle, getattr(pp, "PP_KERNEL_" + kernel))
         xd = dev(x)
         outs = []
         for _ in range(5):
@@ -167,7 +216,7 @@ def test_autotune_keeps_parity(pp, runner, oracle_mod):
     dl = runner.DeviceLayer(L)
     try:
         pp.pp_layer_autotune(dl.handle, 1, 24, 40, pp.PP_RELU, None)
-        assert pp.pp_layer_kernel(dl.handle) in (pp.PP_KERNEL_TC, pp.PP_KERNEL_TMEM)
+        assert pp.pp_layer_kernel(dl.handle) in (pp.PP_KERNEL_TC, pp.PP_KERNEL_TC_FLAT, pp.PP_KERNEL_TMEM)
         y = torch.empty((1, 96, 24, 40), device="cuda")
         dl.forward(dev(x), y, None, 1, 24, 40, pp.PP_RELU, torch.cuda.current_stream())
         torch.cuda.synchronize()
