@@ -144,6 +144,29 @@ pp_status pp_layer_info(const pp_layer* layer, int* Co, int* Ci, int64_t* device
 pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H, int W,
                           int flags, void* stream);
 
+/*
+ * Allocation-free variant of pp_conv_forward for the flat tensor-core kernel
+ * (PP_KERNEL_TC_FLAT).  The paper has no counterpart: it exists for callers
+ * that must not allocate device memory while they run layers (their device
+ * memory budget is reserved up front by another allocator, or their loop
+ * cannot take the device-wide synchronisation that cudaMalloc / cudaFree may
+ * cause), whereas pp_conv_forward grows the layer's split workspace on first
+ * use.  Here the split partials live in one static device array of 16 MiB per
+ * device; no call allocates or frees device memory.
+ *   Runs the flat kernel whatever kernel the layer has selected; same
+ *   arguments, layout, epilogue and fp32 bound as pp_conv_forward.
+ *   The first call on a device looks up the static array's address
+ *   (cudaGetSymbolAddress) and should come before any stream capture.
+ *   The array is shared by every call on the device: calls that overlap in
+ *   time (other streams, other host threads) race on it and must not be made.
+ *   Nothing in the array needs to start at zero.
+ * Errors: as pp_conv_forward; PP_ERR_UNSUPPORTED also when the layer cannot
+ *   run the flat kernel at this shape (Ci < 8, Co <= 64, W > 128) or the
+ *   launch would need more than 16 MiB of split partials.
+ */
+pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H,
+                                  int W, int flags, void* stream);
+
 /* Which kernel pp_conv_forward runs for a layer.  All compute the same
  * convolution within the documented fp32 bound.
  *   PP_KERNEL_TC        implicit GEMM on the tensor cores over the 9 taps

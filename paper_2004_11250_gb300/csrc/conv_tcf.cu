@@ -647,6 +647,9 @@ bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_
   return true;
 }
 
+pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
+                     const float* x, float* y, const float* skip, int N, int H, int W, int flags, cudaStream_t stream);
+
 }  // namespace
 
 namespace ppc {
@@ -684,6 +687,16 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
       if (!ok && !flat_geometry(N, H, W, T.nch, T.nfb, pool, false, *D, &G)) return PP_ERR_UNSUPPORTED;
     }
   }
+  return launch_geo(G, G.split > 1 ? T.scratch->p : nullptr, *D, T, M, x, y, skip, N, H, W, flags, stream);
+}
+
+}  // namespace ppc
+
+namespace {
+
+pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
+                     const float* x, float* y, const float* skip, int N, int H, int W, int flags, cudaStream_t stream) {
+  const DeviceState* D = &Dref;
   FlatParams p;
   p.x = x;
   p.y = y;
@@ -692,7 +705,7 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
   p.perm = M.perm;
   p.bias = M.bias;
   p.status = T.status;
-  p.ws = G.split > 1 ? T.scratch->p : nullptr;
+  p.ws = ws;
   p.N = N;
   p.Ci = M.Ci;
   p.Co = M.Co;
@@ -751,6 +764,43 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
     return PP_ERR_CUDA;
   }
   return PP_OK;
+}
+
+// Split workspace of the allocation-free entry point: one per device, shared
+// by every call on it.  Nothing in it needs to start at zero (each CTA writes
+// its whole partial tile before any CTA of its cluster reads it).
+constexpr size_t STATIC_WS_BYTES = (size_t)16 << 20;
+__device__ __align__(256) float g_static_ws[STATIC_WS_BYTES / sizeof(float)];
+float* g_static_ws_ptr[64] = {};
+
+}  // namespace
+
+namespace ppc {
+
+pp_status tcf_launch_static(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
+                            int H, int W, int flags, cudaStream_t stream) {
+  if (T.FB != FB) return PP_ERR_UNSUPPORTED;
+  DeviceState* D = prepare();
+  if (!D) return PP_ERR_CUDA;
+  FlatGeo G;
+  if (!flat_geometry(N, H, W, T.nch, T.nfb, flags & PP_POOL2, true, *D, &G)) return PP_ERR_UNSUPPORTED;
+  float* ws = nullptr;
+  if (G.split > 1) {
+    if ((size_t)G.ntiles * G.split * FB * G.ncols * sizeof(float) > STATIC_WS_BYTES) return PP_ERR_UNSUPPORTED;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return PP_ERR_CUDA;
+    if (!g_static_ws_ptr[dev]) {
+      // once per device: the address of the static workspace
+      void* a = nullptr;
+      if (cudaGetSymbolAddress(&a, g_static_ws) != cudaSuccess || !a) {
+        cudaGetLastError();
+        return PP_ERR_CUDA;
+      }
+      g_static_ws_ptr[dev] = static_cast<float*>(a);
+    }
+    ws = g_static_ws_ptr[dev];
+  }
+  return launch_geo(G, ws, *D, T, M, x, y, skip, N, H, W, flags, stream);
 }
 
 }  // namespace ppc

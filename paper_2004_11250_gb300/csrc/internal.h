@@ -75,6 +75,10 @@ void tc_free(TcLayout* T);
 // PP_ERR_UNSUPPORTED for shapes it does not handle.
 pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
                      int H, int W, int flags, cudaStream_t stream);
+// The same kernel with its split workspace in a fixed-size static device array
+// instead of the layer's (see pp_conv_forward_noalloc); never allocates.
+pp_status tcf_launch_static(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip,
+                            int N, int H, int W, int flags, cudaStream_t stream);
 
 // True when every pattern of the set is one of the ring patterns (centre plus
 // 3 consecutive neighbours); ring_of[p] receives its ring index.

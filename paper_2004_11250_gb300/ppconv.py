@@ -59,6 +59,7 @@ _SIGS = {
     "pp_layer_create": ([_P, _P, _P, _PP], _I),
     "pp_layer_info": ([_P, _P, _P, _P], _I),
     "pp_conv_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
+    "pp_conv_forward_noalloc": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
     "pp_layer_set_kernel": ([_P, _I], _I),
     "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_device_status": ([_P, _P], _I),
@@ -207,6 +208,12 @@ def pp_layer_info(layer):
 def pp_conv_forward(layer, x, y, skip, N, H, W, flags, stream=None):
     _check(lib.pp_conv_forward(layer, _dp(x), _dp(y), _dp(skip), N, H, W, flags, _stream(stream)),
            "pp_conv_forward")
+
+
+def pp_conv_forward_noalloc(layer, x, y, skip, N, H, W, flags, stream=None):
+    """pp_conv_forward through the flat tensor-core kernel with a static split workspace (no device allocation)."""
+    _check(lib.pp_conv_forward_noalloc(layer, _dp(x), _dp(y), _dp(skip), N, H, W, flags, _stream(stream)),
+           "pp_conv_forward_noalloc")
 
 
 def pp_layer_set_kernel(layer, kernel: int):
