@@ -133,7 +133,9 @@ template <int ORI, int TW, int FB>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p, const __grid_constant__ CUtensorMap xmap) {
   using G = Geo<ORI, TW, FB>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // Offset from the shared array itself (not an integer round trip), so the
+  // compiler keeps every access below in the shared state space.
+  unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t full[2], wfull[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;

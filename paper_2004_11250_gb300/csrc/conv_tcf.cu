@@ -60,17 +60,15 @@ constexpr int WMAX = 128;             // widest map handled
 constexpr int W_TILE = FB * KC * 4;   // one tap, hi or lo: 128 x 8 fp32
 constexpr int W_BYTES = NTAP * 2 * W_TILE;
 constexpr int PIX_MAX = 544;          // staged pixels per K half, padding included
-constexpr int IN_HALF_MAX = PIX_MAX * 16;
-constexpr int IN_MAX = 2 * IN_HALF_MAX;  // hi (or lo) operand of one chunk
-constexpr int LO_MAX = IN_MAX;        // lo operand; the raw tensor-map box lands here first
-constexpr int STAGE = W_BYTES + IN_MAX + LO_MAX;
-constexpr int SMEM_ALLOC = 2 * STAGE + 1024;
+constexpr int IN_MAX = 2 * PIX_MAX * 16;  // largest hi (or lo) operand of one chunk
+constexpr int SMEM_ALLOC = 231424;    // dynamic shared memory (static use stays below 1 KB)
+constexpr int SMEM_USE = SMEM_ALLOC - 1024;  // after aligning the base to 1024
 constexpr int ITEMS_MAX = (2 * PIX_MAX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
-constexpr int PF_AHEAD = 6;           // chunks whose operands are prefetched into L2 ahead of use
+constexpr int PF_AHEAD = 16;          // first chunks whose operands are prefetched into L2
 constexpr long WAIT_LIMIT = 1L << 22;
 constexpr int MAX_SPLIT = 16;
-static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
-static_assert(STAGE % 128 == 0 && (W_BYTES + IN_MAX) % 128 == 0, "stage alignment");
+static_assert(2 * (W_BYTES + 2 * IN_MAX) <= SMEM_USE, "shared memory plan");
+static_assert(FB * NMAX * 4 <= SMEM_USE, "split reduction buffer");
 
 struct FlatParams {
   const float* x;
@@ -84,6 +82,8 @@ struct FlatParams {
   int N, Ci, Co, H, W;
   int nch, nfb, flags, use_tma;
   int bcols, R, ncols, npix, npixa, raw_w, raw_bytes;
+  int stage, lo_off;        // bytes per stage; offset of the lo operand in a stage (hi is at W_BYTES)
+  int sep, raw_off, raw_slot;  // input boxes in a ring of their own (two slots at raw_off)
   int tiles_y, ntiles, split;
   uint32_t idesc;
 };
@@ -102,8 +102,10 @@ __device__ __forceinline__ Tile tile_of(const FlatParams& p, int t) {
 
 template <bool SPLIT>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
-  extern __shared__ __align__(1024) unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  extern __shared__ unsigned char smem_raw[];
+  // Offset from the shared array itself (not an integer round trip), so the
+  // compiler keeps every access below in the shared state space.
+  unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t full[2], wfull[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar, red_bar;
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
@@ -165,25 +167,42 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   if (warp < MMA_WARP) {
     // ------------------------------------------------------------ loaders
     // Chunk sequence g = 0 .. nall-1 of this CTA (tiles in order, each over the
-    // CTA's chunk range).  Thread 0 keeps the weights (and input boxes) of the
-    // next PF_AHEAD chunks on their way into L2, so the copies into shared
-    // memory, which wait for a free stage, find them there.
+    // CTA's chunk range).
     const int nchm = c_end - c_beg;
     const int nall = nmine * nchm;
-    auto prefetch = [&](int gg) {  // thread 0 only
+    // Each loader thread's (K half, pixel) items are the same for every chunk:
+    // their offsets in the input box and in the operand tiles are computed once.
+    int roff[ITEMS_MAX], doff[ITEMS_MAX], rowcol[ITEMS_MAX];
+#pragma unroll
+    for (int b = 0; b < ITEMS_MAX; ++b) {
+      const int it = b * NLOAD + tid;
+      const int kh = it >= p.npix ? 1 : 0;
+      const int pix = it - kh * p.npix;
+      const int br = pix / p.bcols, bc = pix - br * p.bcols;
+      const bool has = it < 2 * p.npix;
+      roff[b] = has ? (kh * 4 * brows + br) * p.raw_w + bc + 3 : -1;
+      doff[b] = has ? kh * p.npixa + pix : -1;
+      rowcol[b] = (kh << 30) | (br << 15) | bc;
+    }
+    const int cstride = brows * p.raw_w;  // between two channels of the box
+    // Input box of chunk gg (thread 0): [8 channels][rows r0-1 ..][columns -4 ..];
+    // zero fill outside the image is the convolution's padding.
+    auto issue_raw = [&](int gg, unsigned char* dst) {
       const int i = gg / nchm, c = c_beg + gg % nchm;
       const Tile T = tile_of(p, tile_index(i));
-      const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(W_BYTES) : "memory");
-      if (p.use_tma)
-        asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
-                         reinterpret_cast<uint64_t>(&xmap)),
-                     "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n)
-                     : "memory");
+      mbar_arrive_expect_tx(su32(&raw_full[gg & 1]), (uint32_t)p.raw_bytes);
+      asm volatile(
+          "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+          "%4, %5}], [%6];" ::"r"(su32(dst)),
+          "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
+          "r"(su32(&raw_full[gg & 1]))
+          : "memory");
     };
-    if (tid == 0)
-      for (int gg = 0; gg < PF_AHEAD && gg < nall; ++gg) prefetch(gg);
+    // With a ring of their own the boxes are copied two chunks ahead of use,
+    // not only once the chunk's stage is free.
     int g = 0, w_issued = 0, raw_issued = 0;
+    if (tid == 0 && p.use_tma && p.sep)
+      for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + p.raw_off + raw_issued * p.raw_slot);
     bool stop = false;  // identical in every loader thread (decided by group_any)
     for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, tile_index(i));
@@ -196,12 +215,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         if (!p.use_tma) {
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b) {
-            const int it = b * NLOAD + tid;
-            const int kh = it >= p.npix ? 1 : 0;
-            const int pix = it - kh * p.npix;
-            const int br = pix / p.bcols, bc = pix - br * p.bcols;
+            const int kh = rowcol[b] >> 30, br = (rowcol[b] >> 15) & 0x7FFF, bc = rowcol[b] & 0x7FFF;
             const int r = T.r0 - 1 + br, cc = bc - 1;
-            const bool inside = it < 2 * p.npix && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
+            const bool inside = doff[b] >= 0 && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               const int ch = c * KC + kh * 4 + k;
@@ -213,9 +229,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           stop = true;
           break;
         }
-        unsigned char* st = smem + s * STAGE;
+        unsigned char* st = smem + (size_t)s * p.stage;
         float4* hi = reinterpret_cast<float4*>(st + W_BYTES);
-        float4* lo = reinterpret_cast<float4*>(st + W_BYTES + IN_MAX);
+        float4* lo = reinterpret_cast<float4*>(st + p.lo_off);
         if (tid == 0) {
           const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
           mbar_arrive_expect_tx(su32(&wfull[s]), W_BYTES);
@@ -224,44 +240,35 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
               "l"(src), "r"(W_BYTES), "r"(su32(&wfull[s]))
               : "memory");
           ++w_issued;
-          if (p.use_tma) {
-            // box [8 channels][rows r0-1 ..][columns -4 ..]; zero fill outside the
-            // image is the convolution's padding
-            mbar_arrive_expect_tx(su32(&raw_full[s]), (uint32_t)p.raw_bytes);
-            asm volatile(
-                "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
-                "%4, %5}], [%6];" ::"r"(su32(lo)),
-                "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
-                "r"(su32(&raw_full[s]))
-                : "memory");
+          if (p.use_tma && !p.sep) {
+            issue_raw(g, reinterpret_cast<unsigned char*>(lo));  // lands in the lo operand, split in place below
             ++raw_issued;
           }
-          if (g + PF_AHEAD < nall) prefetch(g + PF_AHEAD);
         }
         if (p.use_tma) {
           if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
             stop = true;
             break;
           }
-          const float* raw = reinterpret_cast<const float*>(lo);
+          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)s * p.raw_slot)
+                                   : reinterpret_cast<const float*>(lo);
 #pragma unroll
-          for (int b = 0; b < ITEMS_MAX; ++b) {
-            const int it = b * NLOAD + tid;
-            const int kh = it >= p.npix ? 1 : 0;
-            const int pix = it - kh * p.npix;
-            const int br = pix / p.bcols, bc = pix - br * p.bcols;
+          for (int b = 0; b < ITEMS_MAX; ++b)
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              v[b][k] = it < 2 * p.npix ? raw[((kh * 4 + k) * brows + br) * p.raw_w + bc + 3] : 0.f;
+            for (int k = 0; k < 4; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+          // A ring slot is rewritten next by a tensor-map copy (async proxy): each
+          // thread orders its reads of the slot before that copy with a proxy fence.
+          if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          group_sync<NLOAD>();  // the whole box is in registers before its buffer is reused
+          if (p.sep && tid == 0 && raw_issued < nall && raw_issued == g + 2) {
+            issue_raw(raw_issued, smem + p.raw_off + (size_t)s * p.raw_slot);
+            ++raw_issued;
           }
-          group_sync<NLOAD>();  // the whole box is in registers before lo is overwritten
         }
 #pragma unroll
         for (int b = 0; b < ITEMS_MAX; ++b) {
-          const int it = b * NLOAD + tid;
-          if (it < 2 * p.npix) {
-            const int kh = it >= p.npix ? 1 : 0;
-            const int dst = kh * p.npixa + it - kh * p.npix;
+          if (doff[b] >= 0) {
+            const int dst = doff[b];
             float4 h;
             h.x = tf32_hi(v[b][0]);
             h.y = tf32_hi(v[b][1]);
@@ -303,12 +310,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             break;
           }
           tm_fence_after();
-          const unsigned char* st = smem + s * STAGE;
+          const unsigned char* st = smem + (size_t)s * p.stage;
           // descriptors hold address / 16 in their low 14 bits (operands lie below
           // 256 KB), so moving an operand by k pixels of 16 bytes adds k
           const uint64_t w0 = smem_desc(su32(st), FB * 16);
           const uint64_t xh0 = smem_desc(su32(st + W_BYTES), (uint32_t)p.npixa * 16);
-          const uint64_t xl0 = smem_desc(su32(st + W_BYTES + IN_MAX), (uint32_t)p.npixa * 16);
+          const uint64_t xl0 = smem_desc(su32(st + p.lo_off), (uint32_t)p.npixa * 16);
           const uint32_t acc0 = c == c_beg ? 0u : 1u;  // the range's first chunk overwrites the accumulators
 #pragma unroll
           for (int t = 0; t < NTAP; ++t) {
@@ -331,6 +338,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
+    if (tid == (EPI_WARP0 + 7) * 32) {
+      // While the loaders start, one epilogue thread (idle until the first
+      // accumulators are ready) sends the weights and input boxes of the CTA's
+      // first chunks on their way into L2.
+      const int nchm = c_end - c_beg;
+      for (int gg = 0; gg < nmine * nchm && gg < PF_AHEAD; ++gg) {
+        const int i = gg / nchm, c = c_beg + gg % nchm;
+        const Tile T = tile_of(p, tile_index(i));
+        const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(W_BYTES) : "memory");
+        if (p.use_tma)
+          asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                           reinterpret_cast<uint64_t>(&xmap)),
+                       "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n)
+                       : "memory");
+      }
+    }
+    __syncwarp();
     const int q = warp & 3;                     // TMEM lane quadrant of this warp
     const int half = (warp - EPI_WARP0) >> 2;   // the two warps of a quadrant share the work
     const bool pool = p.flags & PP_POOL2;
@@ -437,13 +462,27 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // scope (with proxy fences on both sides, as the partials are written by
     // plain stores and read by bulk copies) orders the partial tiles written
     // above before the copies below.
-    __syncwarp();
-    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-    // This CTA finishes filters [m0, m1) of the tile: the S partials of those
-    // rows (contiguous in the workspace) come into shared memory, freed by the
-    // main loop, by one bulk copy each, and are added in rank order.
+    // This CTA finishes filters [m0, m1) of the tile (below).  Epilogue warp w
+    // takes filters m0 + w, m0 + w + 8, ...; lane i of it holds the original
+    // index and bias of its i-th one, fetched now so the loads overlap the
+    // barrier wait.
     const int tile = (int)blockIdx.x / p.split, rank = (int)blockIdx.x % p.split;
     const int m0 = rank * FB / p.split, m1 = (rank + 1) * FB / p.split, nm = m1 - m0;
+    int o_l = -1;
+    float b_l = 0.f;
+    if (warp >= EPI_WARP0) {
+      const int ml = (warp - EPI_WARP0) + (NEPI / 32) * lane;
+      const int jr = tile_of(p, tile).fb * FB + m0 + ml;
+      if (ml < nm && jr < p.Co) {
+        o_l = __ldg(p.perm + jr);
+        b_l = p.bias ? __ldg(p.bias + jr) : 0.f;
+      }
+    }
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+    // The S partials of the CTA's filters (contiguous rows of the workspace)
+    // come into shared memory, freed by the main loop, by one bulk copy each,
+    // and are added in rank order.
     const uint32_t slice = (uint32_t)(nm * p.ncols * 4);
     bool issued = false;  // thread 0: the copies below were issued
     if (tid == 0 && !abort_s) {
@@ -461,52 +500,80 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     }
     // the whole warp takes one branch (every lane runs the vote)
     if (warp >= EPI_WARP0 && __all_sync(0xffffffffu, !abort_s && wait(&red_bar, 0u))) {
-      const int e = tid - EPI_WARP0 * 32;
       const Tile T = tile_of(p, tile);
       const bool pool = p.flags & PP_POOL2;
       const bool relu = p.flags & PP_RELU;
       const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
       const float* buf = reinterpret_cast<const float*>(smem);  // [S][nm][ncols]
       const int sl = nm * p.ncols;
+      const int ew = (tid >> 5) - EPI_WARP0;  // 0 .. 7: one filter per warp at a time
+      // Each lane's output pixels are the same for every filter: lane + 32 k of
+      // the tile's R x W (pooled: R/2 x W/2) pixels, k < 8 (R * W <= 256).  Their
+      // accumulator columns and output offsets are computed once; each filter
+      // then issues all its shared-memory loads before using them.
       const int Ro = pool ? p.R / 2 : p.R, Wo = pool ? p.W / 2 : p.W;
-      const int total = nm * Ro * Wo;
-      for (int idx = e; idx < total; idx += NEPI) {
-        const int cx = idx % Wo;
-        const int t2 = idx / Wo;
-        const int ro = t2 % Ro, ml = t2 / Ro;
-        const int jr = T.fb * FB + m0 + ml;
-        if (jr >= p.Co) continue;
-        const int o = __ldg(p.perm + jr);
-        const float bs = p.bias ? __ldg(p.bias + jr) : 0.f;
+      const int Ho = pool ? p.H / 2 : p.H;
+      const int r0o = pool ? T.r0 / 2 : T.r0;
+      int colk[8], yoffk[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int j = lane + 32 * k;
+        const int ro = j / Wo, cx = j - ro * Wo;
+        const bool ok = j < Ro * Wo && r0o + ro < Ho;
+        colk[k] = pool ? 2 * ro * p.bcols + 2 * cx : ro * p.bcols + cx;
+        yoffk[k] = ok ? (r0o + ro) * Wo + cx : -1;
+      }
+      for (int ml = ew, i = 0; ml < nm; ml += NEPI / 32, ++i) {
+        const int o = __shfl_sync(0xffffffffu, o_l, i);
+        const float bs = __shfl_sync(0xffffffffu, b_l, i);
+        if (o < 0) break;  // warp-uniform; later filters are beyond Co too
         const size_t plane = (size_t)T.n * p.Co + o;
         const float* src = buf + ml * p.ncols;
+        float* yp = p.y + plane * (size_t)Ho * Wo;
+        const float* sp = skip ? skip + plane * (size_t)p.H * p.W : nullptr;
         if (!pool) {
-          const int row = T.r0 + ro;
-          if (row >= p.H) continue;
-          const int col = ro * p.bcols + cx;
-          float v = 0.f;
-          for (int s = 0; s < p.split; ++s) v += src[s * sl + col];
-          v += bs;
-          const size_t yi = (plane * p.H + row) * p.W + cx;
-          if (skip) v += __ldg(skip + yi);
-          if (relu) v = fmaxf(v, 0.f);
-          p.y[yi] = v;
-        } else {
-          const int rr = 2 * ro, row = T.r0 + rr;
-          if (row >= p.H) continue;
-          float mx = 0.f;
+          float acc[8];
 #pragma unroll
-          for (int d = 0; d < 4; ++d) {
-            const int dr = d >> 1, dc = d & 1;
-            const int col = (rr + dr) * p.bcols + 2 * cx + dc;
-            float v = 0.f;
-            for (int s = 0; s < p.split; ++s) v += src[s * sl + col];
-            v += bs;
-            if (skip) v += __ldg(skip + (plane * p.H + row + dr) * p.W + 2 * cx + dc);
-            if (relu) v = fmaxf(v, 0.f);
-            mx = d == 0 ? v : fmaxf(mx, v);
-          }
-          p.y[(plane * (p.H / 2) + row / 2) * (p.W / 2) + cx] = mx;
+          for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+          for (int s = 0; s < p.split; ++s)
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              if (yoffk[k] >= 0) acc[k] += src[s * sl + colk[k]];
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            if (yoffk[k] >= 0) {
+              float v = acc[k] + bs;
+              if (sp) v += __ldg(sp + yoffk[k]);
+              if (relu) v = fmaxf(v, 0.f);
+              yp[yoffk[k]] = v;
+            }
+        } else {
+          float acc[2][4];
+#pragma unroll
+          for (int k = 0; k < 2; ++k)
+#pragma unroll
+            for (int d = 0; d < 4; ++d) acc[k][d] = 0.f;
+          for (int s = 0; s < p.split; ++s)
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+              if (yoffk[k] >= 0)
+#pragma unroll
+                for (int d = 0; d < 4; ++d) acc[k][d] += src[s * sl + colk[k] + (d >> 1) * p.bcols + (d & 1)];
+#pragma unroll
+          for (int k = 0; k < 2; ++k)
+            if (yoffk[k] >= 0) {
+              // full-resolution position of the window's top-left pixel
+              const int po = yoffk[k] / Wo, pc = yoffk[k] - po * Wo;
+              float mx = 0.f;
+#pragma unroll
+              for (int d = 0; d < 4; ++d) {
+                float v = acc[k][d] + bs;
+                if (sp) v += __ldg(sp + (size_t)(2 * po + (d >> 1)) * p.W + 2 * pc + (d & 1));
+                if (relu) v = fmaxf(v, 0.f);
+                mx = d == 0 ? v : fmaxf(mx, v);
+              }
+              yp[yoffk[k]] = mx;
+            }
         }
       }
     }
@@ -581,6 +648,7 @@ DeviceState* prepare() {
 
 struct FlatGeo {
   int bcols = 0, R = 0, ncols = 0, npix = 0, npixa = 0, raw_w = 0, raw_bytes = 0, tiles_y = 0, ntiles = 0, split = 1;
+  int stage = 0, lo_off = 0, sep = 0, raw_off = 0, raw_slot = 0;
   double cost = 1e300;
 };
 
@@ -619,7 +687,14 @@ bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_
     G.raw_bytes = KC * (R + 2) * G.raw_w * 4;
     G.tiles_y = ty;
     const int64_t nt = (int64_t)ty * nfb * N;
-    if (G.npixa > PIX_MAX || G.raw_bytes > LO_MAX || G.ncols > NMAX || nt > INT32_MAX / MAX_SPLIT) continue;
+    const int in_bytes = (2 * G.npixa * 16 + 127) / 128 * 128;
+    G.raw_slot = (G.raw_bytes + 127) / 128 * 128;
+    G.stage = W_BYTES + 2 * in_bytes;
+    G.sep = 2 * G.stage + 2 * G.raw_slot <= SMEM_USE;
+    if (!G.sep) G.stage = W_BYTES + in_bytes + std::max(in_bytes, G.raw_slot);  // the box lands in lo
+    G.lo_off = W_BYTES + in_bytes;
+    G.raw_off = 2 * G.stage;
+    if (G.npixa > PIX_MAX || 2 * G.stage > SMEM_USE || G.ncols > NMAX || nt > INT32_MAX / MAX_SPLIT) continue;
     G.ntiles = (int)nt;
     const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
     const double per_chunk = std::max(std::max(mma, W_BYTES / 48.0), 1500.0);
@@ -721,6 +796,11 @@ pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const
   p.npixa = G.npixa;
   p.raw_w = G.raw_w;
   p.raw_bytes = G.raw_bytes;
+  p.stage = G.stage;
+  p.lo_off = G.lo_off;
+  p.sep = G.sep;
+  p.raw_off = G.raw_off;
+  p.raw_slot = G.raw_slot;
   p.tiles_y = G.tiles_y;
   p.ntiles = G.ntiles;
   p.split = G.split;
