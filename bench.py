@@ -11,8 +11,11 @@ Printed JSON line (rank 0):
   ms_per_step  ms per frame
   e2e        the same metric through pp_net_run_host (pinned host buffers,
              H2D + run + D2H + sync every step)
-  roofline   the pruned-conv kernel: achieved TFLOP/s over its launches vs the
-             FP32 FMA peak 152 SM x 128 lanes x 2 FLOP x 2.07 GHz
+  roofline   the pruned convs: surviving-weight TFLOP/s over their launches vs
+             the FP32 FMA peak 152 SM x 128 lanes x 2 FLOP x 2.07 GHz (the
+             method's roofline); "tensor" adds the tensor-pipe view of the ops
+             that run on the tensor cores (3xTF32 dense-tap FLOPs executed vs
+             the measured bf16 peak x the nominal tf32 / bf16 ratio)
   cpu_baseline the fp64 CPU oracle on this host's cores on a bounded sample
   configs    ms/frame, GFLOP/s and roofline fraction of all five workloads
 
@@ -38,6 +41,9 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 HBM_PEAK_GBS_FALLBACK = 6800.0
+BF16_PEAK_TFLOPS_FALLBACK = 1900.0
+TF32_PER_BF16 = 1.1 / 2.25  # nominal dense tensor rates
+KERNEL_NAMES = {1: "ppconv_tm_kernel", 2: "ppconv_kernel", 3: "ppconv_tc_kernel", 4: "ppconv_tcf_kernel"}
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
@@ -251,11 +257,19 @@ def traffic_from_profile(kernel_hash: str):
         return None
 
 
+def bf16_peak_tflops():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return BF16_PEAK_TFLOPS_FALLBACK, "fallback"
+
+
 def kernel_source_hash():
     """sha256 over the conv kernel sources (a profile taken on other sources is stale)."""
     import hashlib
     h = hashlib.sha256()
-    for name in ("conv.cu", "conv_tm.cu", "internal.h"):
+    for name in ("conv.cu", "conv_tm.cu", "conv_tc.cu", "conv_tcf.cu", "tc_ptx.cuh", "internal.h"):
         with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()
@@ -279,7 +293,9 @@ def bench_config(name, steps, warmup, flush, stream, hbm):
         fr = [roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3) for s, t in zip(shapes, op_ms)]
         pr = [f for s, f in zip(shapes, fr) if s["pruned"]]
         del acts
-        return {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1),
+        from paper_2004_11250_gb300 import ppconv as pp
+        kern = sorted(set(KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") for L in dn.layers if not L.dense))
+        return {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1), "kernels": kern,
                 "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
                 "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None}
     finally:
@@ -393,6 +409,9 @@ def main():
     ap.add_argument("--no-configs", action="store_true", help="skip the all-configs table")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--kernels", default="",
+                    help="comma list, one per op (tm, reg, tc, flat, or auto to keep the autotuned choice): pins "
+                         "each op's kernel after pp_net_finalize, e.g. to profile the selection of an earlier run")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     ws, rank, local = dist_setup(args)
@@ -413,6 +432,16 @@ def main():
     shapes = op_shapes(spec)
     flops_frame = sum(s["flops"] for s in shapes)
     dn = runner.DeviceNet(spec, use_graph=True)
+    if args.kernels:
+        from paper_2004_11250_gb300 import ppconv as pp
+        ids = {"tm": pp.PP_KERNEL_TMEM, "reg": pp.PP_KERNEL_REGISTER, "tc": pp.PP_KERNEL_TC,
+               "flat": pp.PP_KERNEL_TC_FLAT}
+        names = args.kernels.split(",")
+        if len(names) != len(dn.layers):
+            raise SystemExit(f"--kernels needs {len(dn.layers)} entries")
+        for L, k in zip(dn.layers, names):
+            if k != "auto" and not L.dense:
+                pp.pp_layer_set_kernel(L.handle, ids[k])
     x = torch.from_numpy(spec.x).cuda()
     y = torch.empty(dn.out_shape, device="cuda")
     torch.cuda.synchronize()
@@ -444,6 +473,22 @@ def main():
     kf = sum(shapes[k]["flops"] for k in pruned)
     kt = sum(op_ms[k] for k in pruned) * 1e-3
     achieved = kf / kt / 1e12
+    # which kernel each op runs (autotuned by pp_net_finalize) and the tensor-pipe view
+    from paper_2004_11250_gb300 import ppconv as pp
+    kern = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "ppconv_kernel (dense)"
+            for L in dn.layers]
+    tc_ops = [k for k in pruned if kern[k] in ("ppconv_tc_kernel", "ppconv_tcf_kernel")]
+    tensor = None
+    if tc_ops:
+        # 3 tf32 products per dense tap MAC: hi*hi, lo*hi, hi*lo
+        tf = sum(3 * 2 * shapes[k]["N"] * shapes[k]["Ci"] * shapes[k]["Co"] * 9 * shapes[k]["H"] * shapes[k]["W"]
+                 for k in tc_ops)
+        tt = sum(op_ms[k] for k in tc_ops) * 1e-3
+        bpk, bsrc = bf16_peak_tflops()
+        tpk = bpk * TF32_PER_BF16
+        tensor = {"bound": "tensor", "ops": len(tc_ops), "achieved": round(tf / tt / 1e12, 2), "peak": round(tpk, 1),
+                  "unit": "TFLOP/s (tf32, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
+                  "peak_source": f"{bsrc} bf16 {bpk} TFLOP/s x nominal tf32/bf16 {TF32_PER_BF16:.3f}"}
     traffic = traffic_from_profile(kernel_source_hash())
     layer_fracs = [round(roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3), 3) for s, t in zip(shapes, op_ms)]
 
@@ -488,10 +533,12 @@ def main():
             "gpu_launches": len(spec.ops) * args.steps,
             "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
                          "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
-                         "kernel": "ppconv_tm_kernel / ppconv_kernel (pattern-pruned conv, all pruned ops of a step)",
+                         "kernel": "all pruned ops of a step: " + ", ".join(sorted(set(kern[k] for k in pruned))),
+                         "tensor": tensor,
                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
                          "hbm_peak_gbs": hbm, "hbm_peak_source": hbm_src},
             "layer_roofline_frac": layer_fracs,
+            "layer_kernels": kern,
             "clocks": clk,
             "cpu_baseline": cpu,
             "configs": configs,
