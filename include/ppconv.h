@@ -199,7 +199,9 @@ pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
 pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
 /* Time every kernel that can run this layer on zero-filled scratch tensors of
  * the given shape and flags (a few launches each, on stream, synchronous) and
- * keep the fastest for the layer.  The kernels differ in speed by layer shape:
+ * keep the fastest for the layer; the flat tensor-core kernel is timed at the
+ * best few tile geometries (rows per tile, cluster split) of its cost model and
+ * keeps the winning one for launches of this shape.  The kernels differ in speed by layer shape:
  * the tensor-core kernel needs many output tiles to fill the GPU, the FMA
  * kernels split small layers across thread-block clusters.  Allocates and
  * frees scratch device memory; must not be called during stream capture.

@@ -721,13 +721,22 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
   if (flags & ~(PP_ADD_SKIP | PP_RELU | PP_POOL2)) return PP_ERR_INVALID_ARG;
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   cudaStream_t stream = (cudaStream_t)stream_;
-  std::vector<int> cand;
-  if (L->tc_ok) cand.push_back(PP_KERNEL_TC);
-  if (L->tc_ok && L->tc.FB == 128) cand.push_back(PP_KERNEL_TC_FLAT);
-  if (L->tm_ok) cand.push_back(PP_KERNEL_TMEM);
-  if (cand.empty()) cand.push_back(PP_KERNEL_REGISTER);
+  // Candidates: (kernel, flat-kernel rows per tile, split); the flat kernel is
+  // tried at the few best geometries of its cost model.
+  struct Cand {
+    int kernel, R, S;
+  };
+  std::vector<Cand> cand;
+  if (L->tc_ok) cand.push_back({PP_KERNEL_TC, 0, 0});
+  if (L->tc_ok && L->tc.FB == 128) {
+    int R[4], S[4];
+    const int n = ppc::tcf_plan(L->tc, N, H, W, flags, R, S, 4);
+    for (int k = 0; k < n; ++k) cand.push_back({PP_KERNEL_TC_FLAT, R[k], S[k]});
+  }
+  if (L->tm_ok) cand.push_back({PP_KERNEL_TMEM, 0, 0});
+  if (cand.empty()) cand.push_back({PP_KERNEL_REGISTER, 0, 0});
   if (cand.size() == 1) {
-    L->kernel = cand[0];
+    L->kernel = cand[0].kernel;
     return PP_OK;
   }
   const size_t in_elems = (size_t)N * L->Ci * H * W, out_elems = (size_t)N * L->Co * H * W;
@@ -746,11 +755,12 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (st == PP_OK && (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess)) st = PP_ERR_CUDA;
   const int saved = L->kernel;
-  int best = saved;
+  Cand best = {saved, 0, 0};
   float best_ms = 1e30f;
-  for (int k : cand) {
+  for (const Cand& c : cand) {
     if (st != PP_OK) break;
-    L->kernel = k;
+    L->kernel = c.kernel;
+    if (c.kernel == PP_KERNEL_TC_FLAT) ppc::tcf_pin(L->tc, N, H, W, flags, c.R, c.S);
     for (int w = 0; w < 2 && st == PP_OK; ++w) st = launch(L, x, y, sk, N, H, W, flags, stream);
     if (st != PP_OK) break;
     if (cudaEventRecord(e0, stream) != cudaSuccess) {
@@ -766,10 +776,13 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
     }
     if (ms < best_ms) {
       best_ms = ms;
-      best = k;
+      best = c;
     }
   }
-  L->kernel = st == PP_OK ? best : saved;
+  L->kernel = st == PP_OK ? best.kernel : saved;
+  // the flat kernel keeps the geometry that won for this shape (none if it lost)
+  if (L->tc_ok && L->tc.FB == 128)
+    ppc::tcf_pin(L->tc, N, H, W, flags, st == PP_OK && best.kernel == PP_KERNEL_TC_FLAT ? best.R : 0, best.S);
   if (e0) cudaEventDestroy(e0);
   if (e1) cudaEventDestroy(e1);
   cudaStreamSynchronize(stream);

@@ -660,14 +660,16 @@ struct FlatGeo {
 // staging latency with two stages; a start-up and pipeline fill of ~5000
 // cycles; the split's partial-tile round trip through L2 at ~64 bytes per
 // cycle; and clusters beyond those co-resident on the GPU run in later waves.
-bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
-                   FlatGeo* out) {
-  if (W < 1 || W > WMAX || H < 1) return false;
+// Every geometry the kernel can run for this shape, best first by the model;
+// fills up to maxn entries and returns how many.
+int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
+                    FlatGeo* out, int maxn) {
+  if (W < 1 || W > WMAX || H < 1 || maxn < 1) return 0;
   const int bcols = (W + 2 + 7) / 8 * 8;
   const int rmax = NMAX / bcols;
-  if (rmax < 1 || (pool && rmax < 2)) return false;
-  FlatGeo best;
-  for (int r0 = rmax; r0 >= 1; r0 = r0 / 2) {
+  if (rmax < 1 || (pool && rmax < 2)) return 0;
+  int n = 0;
+  for (int r0 = rmax; r0 >= 1; --r0) {
     int R = std::min(r0, H);
     int ty = (H + R - 1) / R;
     R = (H + ty - 1) / ty;  // balance the rows over the tiles
@@ -709,17 +711,46 @@ bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_
         const double waves = std::ceil((double)G.ntiles / D.max_clusters[s]);
         cost = waves * (std::ceil((double)nch / s) * per_chunk + 5000.0 + 16.0 * G.ncols);
       }
-      if (cost < best.cost) {
-        best = G;
-        best.split = s;
-        best.cost = cost;
+      G.split = s;
+      G.cost = cost;
+      bool dup = false;
+      for (int k = 0; k < n; ++k) dup = dup || (out[k].R == G.R && out[k].split == s);
+      if (dup) continue;
+      // insert in cost order, keeping the best maxn
+      if (n == maxn && out[n - 1].cost <= cost) continue;
+      int k = n < maxn ? n++ : maxn - 1;  // a full list drops its worst entry
+      while (k > 0 && out[k - 1].cost > cost) {
+        out[k] = out[k - 1];
+        --k;
       }
+      out[k] = G;
     }
-    if (r0 == 1) break;
   }
-  if (best.R == 0) return false;
-  *out = best;
-  return true;
+  return n;
+}
+
+bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
+                   FlatGeo* out) {
+  return flat_candidates(N, H, W, nch, nfb, pool, allow_split, D, out, 1) == 1;
+}
+
+// The geometry (R, split) for this shape if the model can run it.
+bool flat_pick(int N, int H, int W, int nch, int nfb, bool pool, const DeviceState& D, int R, int S, FlatGeo* out) {
+  FlatGeo all[160];
+  const int n = flat_candidates(N, H, W, nch, nfb, pool, true, D, all, 160);
+  for (int k = 0; k < n; ++k)
+    if (all[k].R == R && all[k].split == S) {
+      *out = all[k];
+      return true;
+    }
+  return false;
+}
+
+// The geometry pinned by timing for this shape, if any.
+bool pinned_geometry(const ppc::TcLayout& T, int N, int H, int W, int flags, const DeviceState& D, FlatGeo* out) {
+  const ppc::TcScratch* st = T.scratch;
+  if (!st || st->R <= 0 || st->key[0] != N || st->key[1] != H || st->key[2] != W || st->key[3] != flags) return false;
+  return flat_pick(N, H, W, T.nch, T.nfb, flags & PP_POOL2, D, st->R, st->S, out);
 }
 
 pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
@@ -736,7 +767,8 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
   if (!D) return PP_ERR_CUDA;
   const bool pool = flags & PP_POOL2;
   FlatGeo G;
-  if (!flat_geometry(N, H, W, T.nch, T.nfb, pool, true, *D, &G)) return PP_ERR_UNSUPPORTED;
+  if (!pinned_geometry(T, N, H, W, flags, *D, &G) && !flat_geometry(N, H, W, T.nch, T.nfb, pool, true, *D, &G))
+    return PP_ERR_UNSUPPORTED;
   if (G.split > 1) {
     const size_t need = (size_t)G.ntiles * G.split * FB * G.ncols * sizeof(float);
     if (T.scratch->bytes < need) {
@@ -857,13 +889,39 @@ float* g_static_ws_ptr[64] = {};
 
 namespace ppc {
 
+int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, int maxn) {
+  if (T.FB != FB || maxn < 1) return 0;
+  DeviceState* D = prepare();
+  if (!D) return 0;
+  FlatGeo G[16];
+  const int n = flat_candidates(N, H, W, T.nch, T.nfb, flags & PP_POOL2, true, *D, G, std::min(maxn, 16));
+  for (int k = 0; k < n; ++k) {
+    R[k] = G[k].R;
+    S[k] = G[k].split;
+  }
+  return n;
+}
+
+void tcf_pin(const TcLayout& T, int N, int H, int W, int flags, int R, int S) {
+  if (!T.scratch) return;
+  TcScratch* st = T.scratch;
+  st->key[0] = N;
+  st->key[1] = H;
+  st->key[2] = W;
+  st->key[3] = flags;
+  st->R = R;
+  st->S = S;
+}
+
 pp_status tcf_launch_static(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
                             int H, int W, int flags, cudaStream_t stream) {
   if (T.FB != FB) return PP_ERR_UNSUPPORTED;
   DeviceState* D = prepare();
   if (!D) return PP_ERR_CUDA;
   FlatGeo G;
-  if (!flat_geometry(N, H, W, T.nch, T.nfb, flags & PP_POOL2, true, *D, &G)) return PP_ERR_UNSUPPORTED;
+  if (!pinned_geometry(T, N, H, W, flags, *D, &G) &&
+      !flat_geometry(N, H, W, T.nch, T.nfb, flags & PP_POOL2, true, *D, &G))
+    return PP_ERR_UNSUPPORTED;
   float* ws = nullptr;
   if (G.split > 1) {
     if ((size_t)G.ntiles * G.split * FB * G.ncols * sizeof(float) > STATIC_WS_BYTES) return PP_ERR_UNSUPPORTED;

@@ -52,6 +52,10 @@ struct TmLayout {
 struct TcScratch {
   float* p = nullptr;
   size_t bytes = 0;
+  // Flat-kernel geometry chosen by timing (pp_layer_autotune) for one shape:
+  // rows per tile and split, used while (N, H, W, flags) match key.
+  int key[4] = {0, 0, 0, -1};
+  int R = 0, S = 0;
 };
 
 // Dense per-tap tf32 hi/lo weight tiles of the tensor-core kernels (conv_tc.cu,
@@ -75,6 +79,11 @@ void tc_free(TcLayout* T);
 // PP_ERR_UNSUPPORTED for shapes it does not handle.
 pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
                      int H, int W, int flags, cudaStream_t stream);
+// The flat kernel's best geometries (rows per tile R, split S) for a shape by
+// its cost model, best first; returns how many (up to maxn).
+int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, int maxn);
+// Use geometry (R, S) for launches of this shape (R = 0: back to the model).
+void tcf_pin(const TcLayout& T, int N, int H, int W, int flags, int R, int S);
 // The same kernel with its split workspace in a fixed-size static device array
 // instead of the layer's (see pp_conv_forward_noalloc); never allocates.
 pp_status tcf_launch_static(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip,
