@@ -462,16 +462,16 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // scope (with proxy fences on both sides, as the partials are written by
     // plain stores and read by bulk copies) orders the partial tiles written
     // above before the copies below.
-    // This CTA finishes filters [m0, m1) of the tile (below).  Epilogue warp w
-    // takes filters m0 + w, m0 + w + 8, ...; lane i of it holds the original
-    // index and bias of its i-th one, fetched now so the loads overlap the
-    // barrier wait.
+    // This CTA finishes filters [m0, m1) of the tile (below), with all its
+    // warps: warp w takes filters m0 + w, m0 + w + 17, ...; lane i of it holds
+    // the original index and bias of its i-th one, fetched now so the loads
+    // overlap the barrier wait.
     const int tile = (int)blockIdx.x / p.split, rank = (int)blockIdx.x % p.split;
     const int m0 = rank * FB / p.split, m1 = (rank + 1) * FB / p.split, nm = m1 - m0;
     int o_l = -1;
     float b_l = 0.f;
-    if (warp >= EPI_WARP0) {
-      const int ml = (warp - EPI_WARP0) + (NEPI / 32) * lane;
+    {
+      const int ml = warp + (NTHREADS / 32) * lane;
       const int jr = tile_of(p, tile).fb * FB + m0 + ml;
       if (ml < nm && jr < p.Co) {
         o_l = __ldg(p.perm + jr);
@@ -499,14 +499,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       }
     }
     // the whole warp takes one branch (every lane runs the vote)
-    if (warp >= EPI_WARP0 && __all_sync(0xffffffffu, !abort_s && wait(&red_bar, 0u))) {
+    if (__all_sync(0xffffffffu, !abort_s && wait(&red_bar, 0u))) {
       const Tile T = tile_of(p, tile);
       const bool pool = p.flags & PP_POOL2;
       const bool relu = p.flags & PP_RELU;
       const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
       const float* buf = reinterpret_cast<const float*>(smem);  // [S][nm][ncols]
       const int sl = nm * p.ncols;
-      const int ew = (tid >> 5) - EPI_WARP0;  // 0 .. 7: one filter per warp at a time
+      const int ew = warp;  // one filter per warp at a time
       // Each lane's output pixels are the same for every filter: lane + 32 k of
       // the tile's R x W (pooled: R/2 x W/2) pixels, k < 8 (R * W <= 256).  Their
       // accumulator columns and output offsets are computed once; each filter
@@ -523,7 +523,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         colk[k] = pool ? 2 * ro * p.bcols + 2 * cx : ro * p.bcols + cx;
         yoffk[k] = ok ? (r0o + ro) * Wo + cx : -1;
       }
-      for (int ml = ew, i = 0; ml < nm; ml += NEPI / 32, ++i) {
+      for (int ml = ew, i = 0; ml < nm; ml += NTHREADS / 32, ++i) {
         const int o = __shfl_sync(0xffffffffu, o_l, i);
         const float bs = __shfl_sync(0xffffffffu, b_l, i);
         if (o < 0) break;  // warp-uniform; later filters are beyond Co too
