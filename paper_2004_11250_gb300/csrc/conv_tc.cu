@@ -89,7 +89,13 @@ struct TcParams {
 template <int ORI, int TW, int FB>
 struct Geo {
   static_assert(ORI == ORI_FP ? FB == 128 : TW == 128, "orientation needs a 128-row M side");
-  static constexpr int SEGC = ORI == ORI_FP ? TW : FB;   // accumulator columns per row segment
+  // MRG (pixel rows x 64 filters): the hi and lo weight tiles of a tap are one
+  // 128-wide B operand, so x_hi * [w_hi | w_lo] is one N = 128 MMA (the lo part
+  // lands in accumulator columns FB .. 2 FB - 1 and the epilogue adds the two
+  // halves); x_lo * w_hi is an N = 64 MMA.  Two MMAs instead of three read the
+  // pixel tile twice instead of three times.
+  static constexpr bool MRG = ORI == ORI_PF && FB == 64;
+  static constexpr int SEGC = ORI == ORI_FP ? TW : (MRG ? 2 * FB : FB);  // accumulator columns per row segment
   static constexpr int R = NCOL / SEGC;                   // row segments per tile
   static constexpr int BROWS = R + 2, BCOLS = TW + 2;
   static constexpr int NPIX = BROWS * BCOLS;              // staged input pixels
@@ -111,6 +117,8 @@ struct Geo {
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
   static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
   static constexpr uint32_t IDESC = ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB);
+  static constexpr uint32_t IDESC2 = idesc_tf32(128, 2 * FB);  // MRG: [w_hi | w_lo]
+  static constexpr int WLBO = MRG ? 2 * FB * 16 : FB * 16;  // weight tile: bytes between K halves
 };
 
 struct Tile {
@@ -339,7 +347,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           const unsigned char* st = smem + s * G::STAGE;
           // Descriptors hold address / 16 in their low 14 bits and every operand
           // lies below 256 KB, so moving an operand is one add to the descriptor.
-          const uint64_t w0 = smem_desc(su32(st), FB * 16);
+          const uint64_t w0 = smem_desc(su32(st), G::WLBO);
           const uint64_t xh0 = smem_desc(su32(st + G::W_BYTES), G::IN_HALF);
           const uint64_t xl0 = smem_desc(su32(st + G::W_BYTES + G::IN_HALF * 2), G::IN_HALF);
           const uint32_t acc0 = c == 0 ? 0u : 1u;  // the tile's first chunk overwrites the accumulators
@@ -357,6 +365,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
                 mma_tf32(d, whi, xh, G::IDESC, t == 0 ? acc0 : 1u);
                 mma_tf32(d, wlo, xh, G::IDESC, 1u);
                 mma_tf32(d, whi, xl, G::IDESC, 1u);
+              } else if (G::MRG) {
+                mma_tf32(d, xh, whi, G::IDESC2, t == 0 ? acc0 : 1u);
+                mma_tf32(d, xl, whi, G::IDESC, 1u);
               } else {
                 mma_tf32(d, xh, whi, G::IDESC, t == 0 ? acc0 : 1u);
                 mma_tf32(d, xh, wlo, G::IDESC, 1u);
@@ -472,6 +483,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             float a[16], bb[16];
             tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + jj), a);
             if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + jj), bb);
+            if (G::MRG) {
+              float a2[16], bb2[16];
+              tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + FB + jj), a2);
+              if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + FB + jj), bb2);
+              tm_wait_ld();
+#pragma unroll
+              for (int k = 0; k < 16; ++k) {
+                a[k] += a2[k];
+                if (pool) bb[k] += bb2[k];
+              }
+            }
             tm_wait_ld();
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
@@ -597,8 +619,9 @@ pp_status tc_prepare() {
 
 // Dense per-tap weights of every (FB-filter block, 8-channel chunk), split into
 // tf32 hi / lo, in the canonical K-major layout: element (filter f, channel k)
-// of a tile at byte (k / 4) * (FB * 16) + f * 16 + (k % 4) * 4.  FB = 64 for
-// layers with at most 64 filters, else 128.
+// of a tile at byte (k / 4) * (FB * 16) + f * 16 + (k % 4) * 4, the hi tile then
+// the lo tile of each tap.  FB = 64 for layers with at most 64 filters (then a
+// tap's hi and lo are rows 0-63 and 64-127 of one 128-row tile), else 128.
 pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
   const int Co = pk->Co, Ci = pk->Ci;
   const int FB = Co <= 64 ? 64 : 128;
@@ -624,9 +647,17 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
         const float lo = w - hi;
         const int t = taps[s];
         const size_t base = ((size_t)fb * T->nch + c) * wchunk + (size_t)t * 2 * wtile;
-        const size_t within = (size_t)(k / 4) * (FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
-        host[(base + within) / 4] = hi;
-        host[(base + wtile + within) / 4] = lo;
+        if (FB == 64) {
+          // one 128-row tile per tap, rows 0-63 hi and 64-127 lo (the pixel-major
+          // kernel's merged B operand)
+          const size_t within = (size_t)(k / 4) * (2 * FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
+          host[(base + within) / 4] = hi;
+          host[(base + within + FB * 16) / 4] = lo;
+        } else {
+          const size_t within = (size_t)(k / 4) * (FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
+          host[(base + within) / 4] = hi;
+          host[(base + wtile + within) / 4] = lo;
+        }
       }
     }
   }
