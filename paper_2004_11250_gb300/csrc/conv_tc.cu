@@ -89,12 +89,12 @@ struct TcParams {
 template <int ORI, int TW, int FB>
 struct Geo {
   static_assert(ORI == ORI_FP ? FB == 128 : TW == 128, "orientation needs a 128-row M side");
-  // MRG (pixel rows x 64 filters): the hi and lo weight tiles of a tap are one
-  // 128-wide B operand, so x_hi * [w_hi | w_lo] is one N = 128 MMA (the lo part
-  // lands in accumulator columns FB .. 2 FB - 1 and the epilogue adds the two
-  // halves); x_lo * w_hi is an N = 64 MMA.  Two MMAs instead of three read the
-  // pixel tile twice instead of three times.
-  static constexpr bool MRG = ORI == ORI_PF && FB == 64;
+  // MRG (pixel-major): the hi and lo weight tiles of a tap are one 2 FB-wide B
+  // operand, so x_hi * [w_hi | w_lo] is one N = 2 FB MMA (the lo part lands in
+  // accumulator columns FB .. 2 FB - 1 and the epilogue adds the two halves);
+  // x_lo * w_hi is an N = FB MMA.  Two MMAs instead of three read the pixel
+  // tile twice instead of three times.
+  static constexpr bool MRG = ORI == ORI_PF;
   static constexpr int SEGC = ORI == ORI_FP ? TW : (MRG ? 2 * FB : FB);  // accumulator columns per row segment
   static constexpr int R = NCOL / SEGC;                   // row segments per tile
   static constexpr int BROWS = R + 2, BCOLS = TW + 2;
@@ -118,7 +118,7 @@ struct Geo {
   static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
   static constexpr uint32_t IDESC = ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB);
   static constexpr uint32_t IDESC2 = idesc_tf32(128, 2 * FB);  // MRG: [w_hi | w_lo]
-  static constexpr int WLBO = MRG ? 2 * FB * 16 : FB * 16;  // weight tile: bytes between K halves
+  static constexpr int WLBO = 2 * FB * 16;  // weights: bytes between K halves (hi and lo rows of a tap in each)
 };
 
 struct Tile {
@@ -355,7 +355,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           for (int t = 0; t < NTAP; ++t) {
             const int dy = t / 3, dx = t % 3;
             const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * G::W_TILE / 16);
-            const uint64_t wlo = w0 + (uint64_t)((t * 2 + 1) * G::W_TILE / 16);
+            const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows: FB rows of 16 bytes
 #pragma unroll(G::R <= 8 ? G::R : 4)
             for (int rr = 0; rr < G::R; ++rr) {
               const uint64_t off = (uint64_t)((rr + dy) * G::BCOLS + dx);  // pixels of 16 bytes
@@ -618,10 +618,12 @@ pp_status tc_prepare() {
 }
 
 // Dense per-tap weights of every (FB-filter block, 8-channel chunk), split into
-// tf32 hi / lo, in the canonical K-major layout: element (filter f, channel k)
-// of a tile at byte (k / 4) * (FB * 16) + f * 16 + (k % 4) * 4, the hi tile then
-// the lo tile of each tap.  FB = 64 for layers with at most 64 filters (then a
-// tap's hi and lo are rows 0-63 and 64-127 of one 128-row tile), else 128.
+// tf32 hi / lo, in the canonical K-major layout of one 2 FB-row tile per tap
+// (rows 0 .. FB-1 the hi values, FB .. 2 FB-1 the lo values): element (row r,
+// channel k) at byte (k / 4) * (2 FB * 16) + r * 16 + (k % 4) * 4.  The hi or the
+// lo rows alone are an FB-row operand with the same K-half stride; all of them
+// are the pixel-major kernel's merged operand.  FB = 64 for layers with at most
+// 64 filters, else 128.
 pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
   const int Co = pk->Co, Ci = pk->Ci;
   const int FB = Co <= 64 ? 64 : 128;
@@ -647,17 +649,10 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
         const float lo = w - hi;
         const int t = taps[s];
         const size_t base = ((size_t)fb * T->nch + c) * wchunk + (size_t)t * 2 * wtile;
-        if (FB == 64) {
-          // one 128-row tile per tap, rows 0-63 hi and 64-127 lo (the pixel-major
-          // kernel's merged B operand)
-          const size_t within = (size_t)(k / 4) * (2 * FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
-          host[(base + within) / 4] = hi;
-          host[(base + within + FB * 16) / 4] = lo;
-        } else {
-          const size_t within = (size_t)(k / 4) * (FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
-          host[(base + within) / 4] = hi;
-          host[(base + wtile + within) / 4] = lo;
-        }
+        // one 2 FB-row tile per tap: rows 0 .. FB-1 hi, FB .. 2 FB-1 lo
+        const size_t within = (size_t)(k / 4) * (2 * FB * 16) + (size_t)f * 16 + (size_t)(k % 4) * 4;
+        host[(base + within) / 4] = hi;
+        host[(base + within + FB * 16) / 4] = lo;
       }
     }
   }
@@ -685,8 +680,10 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
 }
 
 // Geometry the launch will use: orientation and tile width for a map width.
-void tc_geometry(const TcLayout& T, int W, int* ori, int* tw) {
-  if (T.FB == 64 || W >= 96) {
+void tc_geometry(const TcLayout& T, int W, bool pool, int* ori, int* tw) {
+  // a pixel-major tile with 128 filters holds one output row (its accumulator
+  // row segment is 2 x 128 columns wide), and pooling needs row pairs
+  if ((T.FB == 64 || W >= 96) && !(T.FB == 128 && pool)) {
     *ori = ORI_PF;
     *tw = 128;
   } else {
@@ -717,7 +714,7 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
   p.FB = T.FB;
   p.flags = flags;
   int ori, tw;
-  tc_geometry(T, W, &ori, &tw);
+  tc_geometry(T, W, (flags & PP_POOL2) != 0, &ori, &tw);
   cudaError_t e;
   if (ori == ORI_PF)
     e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, g_sms) : launch<ORI_PF, 128, 128>(p, stream, g_sms);

@@ -313,7 +313,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           const unsigned char* st = smem + (size_t)s * p.stage;
           // descriptors hold address / 16 in their low 14 bits (operands lie below
           // 256 KB), so moving an operand by k pixels of 16 bytes adds k
-          const uint64_t w0 = smem_desc(su32(st), FB * 16);
+          const uint64_t w0 = smem_desc(su32(st), 2 * FB * 16);  // hi and lo rows of a tap in each K half
           const uint64_t xh0 = smem_desc(su32(st + W_BYTES), (uint32_t)p.npixa * 16);
           const uint64_t xl0 = smem_desc(su32(st + p.lo_off), (uint32_t)p.npixa * 16);
           const uint32_t acc0 = c == c_beg ? 0u : 1u;  // the range's first chunk overwrites the accumulators
@@ -321,7 +321,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           for (int t = 0; t < NTAP; ++t) {
             const uint64_t off = (uint64_t)((t / 3) * p.bcols + t % 3);
             const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * W_TILE / 16);
-            const uint64_t wlo = w0 + (uint64_t)((t * 2 + 1) * W_TILE / 16);
+            const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows
             mma_tf32(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
             mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
             mma_tf32(d, whi, xl0 + off, p.idesc, 1u);

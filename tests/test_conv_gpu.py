@@ -130,6 +130,23 @@ def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
         check_within(g, y, s, f"tensor-core kernel {(N, Ci, Co, H, W)}")
 
 
+@pytest.mark.parametrize("shape", [(1, 40, 130, 7, 100), (2, 16, 200, 4, 144), (1, 24, 64, 6, 160)])
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+def test_tensor_core_pixel_major(pp, runner, oracle_mod, shape, flags):
+    """Maps at least 96 wide: the row-tiled kernel's pixel-major tiles (merged hi/lo weight operand), 64- and
+    128-filter blocks, ragged filter blocks and row ends; pooled 128-filter layers take filter-major tiles."""
+    N, Ci, Co, H, W = shape
+    if flags == "pool_relu" and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(13 * sum(shape) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.45)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=pp.PP_KERNEL_TC)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
+    check_within(g, y, s, f"pixel-major tensor-core kernel {shape} {flags}")
+
+
 FLAT_CASES = [
     # N, Ci, Co, H, W: every map width class, ragged filter blocks and channel
     # chunks, tiles that overhang the map, split and persistent launches
