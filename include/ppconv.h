@@ -145,24 +145,19 @@ pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const
                           int flags, void* stream);
 
 /*
- * Allocation-free variant of pp_conv_forward for the flat tensor-core kernel
- * (PP_KERNEL_TC_FLAT).  The paper has no counterpart: it exists for callers
- * that must not allocate device memory while they run layers (their device
- * memory budget is reserved up front by another allocator, or their loop
- * cannot take the device-wide synchronisation that cudaMalloc / cudaFree may
- * cause), whereas pp_conv_forward grows the layer's split workspace on first
- * use.  Here the split partials live in one static device array of 16 MiB per
- * device; no call allocates or frees device memory.
- *   Runs the flat kernel whatever kernel the layer has selected; same
- *   arguments, layout, epilogue and fp32 bound as pp_conv_forward.
- *   The first call on a device looks up the static array's address
- *   (cudaGetSymbolAddress) and should come before any stream capture.
- *   The array is shared by every call on the device: calls that overlap in
- *   time (other streams, other host threads) race on it and must not be made.
- *   Nothing in the array needs to start at zero.
+ * Allocation-free forward through the flat tensor-core kernel
+ * (PP_KERNEL_TC_FLAT).  The paper has no counterpart: it is for callers that
+ * must not allocate device memory while they run layers (their device memory
+ * budget is reserved up front by another allocator, or their loop cannot take
+ * the device-wide synchronisation that cudaMalloc / cudaFree may cause).  The
+ * flat kernel reduces its cluster-split partial tiles through distributed
+ * shared memory, so it needs no workspace; this call runs it whatever kernel
+ * the layer has selected and never allocates or frees device memory.
+ *   Same arguments, layout, epilogue and fp32 bound as pp_conv_forward.
+ *   The first call on a device sets the kernel's launch attributes and should
+ *   come before any stream capture.
  * Errors: as pp_conv_forward; PP_ERR_UNSUPPORTED also when the layer cannot
- *   run the flat kernel at this shape (Ci < 8, Co <= 64, W > 128) or the
- *   launch would need more than 16 MiB of split partials.
+ *   run the flat kernel at this shape (Ci < 8, Co <= 64, W > 128).
  */
 pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H,
                                   int W, int flags, void* stream);
@@ -174,14 +169,10 @@ pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* 
  *                       pattern set; needs Ci >= 8.
  *   PP_KERNEL_TC_FLAT   the same contraction with whole output rows flattened
  *                       into one MMA and, for layers with few output tiles,
- *                       the input channels split over a thread-block cluster;
- *                       maps at most 128 pixels wide and layers with more than
- *                       64 filters (other shapes run PP_KERNEL_TC).  A split
- *                       launch keeps fp32 partial tiles in a workspace owned
- *                       by the layer, allocated on first use outside stream
- *                       capture (inside a capture without one, the launch
- *                       runs unsplit); so calls of one layer must not run
- *                       concurrently on different streams.
+ *                       the input channels split over a thread-block cluster
+ *                       (partial tiles reduced through distributed shared
+ *                       memory); maps at most 128 pixels wide and layers with
+ *                       more than 64 filters (other shapes run PP_KERNEL_TC).
  *   PP_KERNEL_TMEM      FP32 FMA over kept taps only, accumulators in tensor
  *                       memory; ring patterns only (the centre tap plus 3
  *                       consecutive of its 8 neighbours).

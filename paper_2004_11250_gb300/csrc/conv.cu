@@ -814,11 +814,8 @@ extern "C" pp_status pp_conv_forward(const pp_layer* L, const float* x, float* y
   return launch(L, x, y, skip, N, H, W, flags, (cudaStream_t)stream);
 }
 
-// The flat tensor-core kernel with its split partials in a static device
-// array: for callers that must not allocate device memory while they run
-// layers (a device memory budget reserved up front by another allocator, or a
-// loop that cannot take the device-wide synchronisation a cudaMalloc or
-// cudaFree may cause).  See the declaration for the contract.
+// The flat tensor-core kernel, with no device memory allocated by the call
+// (see the declaration).
 extern "C" pp_status pp_conv_forward_noalloc(const pp_layer* L, const float* x, float* y, const float* skip, int N,
                                              int H, int W, int flags, void* stream) {
   if (!L || !x || !y || N < 1 || H < 1 || W < 1) return PP_ERR_INVALID_ARG;
@@ -832,7 +829,7 @@ extern "C" pp_status pp_conv_forward_noalloc(const pp_layer* L, const float* x, 
   M.Ci = L->Ci;
   M.perm = L->perm;
   M.bias = L->has_bias ? L->bias : nullptr;
-  return ppc::tcf_launch_static(L->tc, M, x, y, skip, N, H, W, flags, (cudaStream_t)stream);
+  return ppc::tcf_launch(L->tc, M, x, y, skip, N, H, W, flags, (cudaStream_t)stream);
 }
 
 extern "C" void pp_layer_destroy(pp_layer* L) {

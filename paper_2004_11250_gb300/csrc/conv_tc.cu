@@ -667,8 +667,8 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
     cudaFree(d);
     return PP_ERR_CUDA;
   }
-  T->scratch = new (std::nothrow) TcScratch();
-  if (!T->scratch) {
+  T->state = new (std::nothrow) TcState();
+  if (!T->state) {
     cudaFree(d);
     return PP_ERR_OOM;
   }
@@ -736,11 +736,8 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
 void tc_free(TcLayout* T) {
   if (T->dmem) cudaFree(T->dmem);
   T->dmem = nullptr;
-  if (T->scratch) {
-    if (T->scratch->p) cudaFree(T->scratch->p);
-    delete T->scratch;
-    T->scratch = nullptr;
-  }
+  delete T->state;
+  T->state = nullptr;
 }
 
 pp_status tc_status(const TcLayout& T, int* device_error) {

@@ -20,11 +20,11 @@
 //
 // Split: when the layer has fewer output tiles than SMs, S CTAs of a cluster
 // share a tile, each summing a contiguous range of the channel chunks.  Each
-// writes its fp32 partial tile to a workspace in global memory (it stays in
-// L2), the cluster barrier orders those writes before the reads, and each CTA
-// then finishes 1/S of the tile's filters: bulk copies bring the S partials of
-// those filters into shared memory, where they are added in rank order
-// (deterministic), then bias, skip, ReLU, pool, and y is stored.
+// copies its fp32 partial tile from TMEM into its own shared memory, a cluster
+// barrier orders those writes before the reads, and each CTA then finishes 1/S
+// of the tile's filters: it reads the S partials of those filters through
+// distributed shared memory, adds them in rank order (deterministic), then
+// bias, skip, ReLU, pool, and stores y.  No global workspace is used.
 //
 // Roles (17 warps, one CTA per SM): warps 0-7 stage the operands, warp 8
 // allocates TMEM and one of its threads issues the MMAs, warps 9-16 are the
@@ -33,6 +33,7 @@
 // the next tile's MMAs.  Every mbarrier wait is bounded; a timeout sets the
 // layer's device status word and the CTA skips the rest of its work (every
 // thread still reaches the cluster barrier).
+#include <cooperative_groups.h>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -78,7 +79,6 @@ struct FlatParams {
   const int* perm;
   const float* bias;
   int* status;
-  float* ws;                // split partials [grid][128][ncols]
   int N, Ci, Co, H, W;
   int nch, nfb, flags, use_tma;
   int bcols, R, ncols, npix, npixa, raw_w, raw_bytes;
@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   // Offset from the shared array itself (not an integer round trip), so the
   // compiler keeps every access below in the shared state space.
   unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
-  __shared__ __align__(8) uint64_t full[2], wfull[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar, red_bar;
+  __shared__ __align__(8) uint64_t full[2], wfull[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
 
@@ -133,7 +133,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       mbar_init(su32(&acc_empty[s]), NEPI);
     }
     mbar_init(su32(&done_bar), 1);
-    mbar_init(su32(&red_bar), 1);
     abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -370,17 +369,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NMAX);
       const int m = 32 * q + lane;  // filter within the block = TMEM lane
       if (SPLIT) {
-        // this CTA's partial tile, row m of [128][ncols] at its grid index
-        float* wrow = p.ws + ((size_t)blockIdx.x * FB + m) * p.ncols;
+        // this CTA's partial tile into its own shared memory (free once the
+        // accumulators are ready): row m of [128][ncols + 4], padded so a warp's
+        // 16-byte stores to 32 rows spread over the banks
+        float* prow = reinterpret_cast<float*>(smem) + m * (p.ncols + 4);
         for (int cb = half * 8; cb < p.ncols; cb += 16) {
           float a[8];
           tm_ld8(lanebase + (uint32_t)cb, a);
           tm_wait_ld();
-          *reinterpret_cast<float4*>(wrow + cb) = make_float4(a[0], a[1], a[2], a[3]);
-          *reinterpret_cast<float4*>(wrow + cb + 4) = make_float4(a[4], a[5], a[6], a[7]);
+          *reinterpret_cast<float4*>(prow + cb) = make_float4(a[0], a[1], a[2], a[3]);
+          *reinterpret_cast<float4*>(prow + cb + 4) = make_float4(a[4], a[5], a[6], a[7]);
         }
-        // the partial is read back by bulk copies (async proxy) in other CTAs
-        asm volatile("fence.proxy.async.global;" ::: "memory");
       } else {
         const int jr = T.fb * FB + m;
         const bool valid = jr < p.Co;
@@ -457,15 +456,16 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   }
 
   if (SPLIT) {
-    // Every thread of every CTA of the cluster arrives, also after an early
-    // stop, so the barrier always completes.  Release / acquire at cluster
-    // scope (with proxy fences on both sides, as the partials are written by
-    // plain stores and read by bulk copies) orders the partial tiles written
-    // above before the copies below.
-    // This CTA finishes filters [m0, m1) of the tile (below), with all its
-    // warps: warp w takes filters m0 + w, m0 + w + 17, ...; lane i of it holds
-    // the original index and bias of its i-th one, fetched now so the loads
-    // overlap the barrier wait.
+    // Every thread of every CTA of the cluster arrives at both cluster
+    // barriers, also after an early stop, so they always complete.  The first
+    // (release / acquire at cluster scope) orders every CTA's partial tile in
+    // its shared memory before the reads below; the second keeps each CTA's
+    // shared memory alive until the others have read it.
+    // This CTA finishes filters [m0, m1) of the tile with all its warps: warp w
+    // takes filters m0 + w, m0 + w + 17, ...; lane i of it holds the original
+    // index and bias of its i-th one, fetched now so the loads overlap the
+    // barrier wait.
+    namespace cg = cooperative_groups;
     const int tile = (int)blockIdx.x / p.split, rank = (int)blockIdx.x % p.split;
     const int m0 = rank * FB / p.split, m1 = (rank + 1) * FB / p.split, nm = m1 - m0;
     int o_l = -1;
@@ -480,37 +480,19 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     }
     __syncwarp();
     asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-    // The S partials of the CTA's filters (contiguous rows of the workspace)
-    // come into shared memory, freed by the main loop, by one bulk copy each,
-    // and are added in rank order.
-    const uint32_t slice = (uint32_t)(nm * p.ncols * 4);
-    bool issued = false;  // thread 0: the copies below were issued
-    if (tid == 0 && !abort_s) {
-      issued = true;
-      asm volatile("fence.proxy.async.global;" ::: "memory");
-      mbar_arrive_expect_tx(su32(&red_bar), slice * (uint32_t)p.split);
-      for (int s = 0; s < p.split; ++s) {
-        const float* src = p.ws + (((size_t)tile * p.split + s) * FB + m0) * p.ncols;
-        asm volatile(
-            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                su32(smem + (size_t)s * slice)),
-            "l"(src), "r"(slice), "r"(su32(&red_bar))
-            : "memory");
-      }
-    }
-    // the whole warp takes one branch (every lane runs the vote)
-    if (__all_sync(0xffffffffu, !abort_s && wait(&red_bar, 0u))) {
+    if (!abort_s) {
+      cg::cluster_group cl = cg::this_cluster();
       const Tile T = tile_of(p, tile);
       const bool pool = p.flags & PP_POOL2;
       const bool relu = p.flags & PP_RELU;
       const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
-      const float* buf = reinterpret_cast<const float*>(smem);  // [S][nm][ncols]
-      const int sl = nm * p.ncols;
-      const int ew = warp;  // one filter per warp at a time
+      const int pst = p.ncols + 4;
+      float* part = reinterpret_cast<float*>(smem);
       // Each lane's output pixels are the same for every filter: lane + 32 k of
       // the tile's R x W (pooled: R/2 x W/2) pixels, k < 8 (R * W <= 256).  Their
       // accumulator columns and output offsets are computed once; each filter
-      // then issues all its shared-memory loads before using them.
+      // then issues all its loads of the S partials (rank order, read from the
+      // cluster's shared memories) before using them.
       const int Ro = pool ? p.R / 2 : p.R, Wo = pool ? p.W / 2 : p.W;
       const int Ho = pool ? p.H / 2 : p.H;
       const int r0o = pool ? T.r0 / 2 : T.r0;
@@ -523,22 +505,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         colk[k] = pool ? 2 * ro * p.bcols + 2 * cx : ro * p.bcols + cx;
         yoffk[k] = ok ? (r0o + ro) * Wo + cx : -1;
       }
-      for (int ml = ew, i = 0; ml < nm; ml += NTHREADS / 32, ++i) {
+      for (int ml = warp, i = 0; ml < nm; ml += NTHREADS / 32, ++i) {
         const int o = __shfl_sync(0xffffffffu, o_l, i);
         const float bs = __shfl_sync(0xffffffffu, b_l, i);
         if (o < 0) break;  // warp-uniform; later filters are beyond Co too
         const size_t plane = (size_t)T.n * p.Co + o;
-        const float* src = buf + ml * p.ncols;
+        const int row = (m0 + ml) * pst;
         float* yp = p.y + plane * (size_t)Ho * Wo;
         const float* sp = skip ? skip + plane * (size_t)p.H * p.W : nullptr;
         if (!pool) {
           float acc[8];
 #pragma unroll
           for (int k = 0; k < 8; ++k) acc[k] = 0.f;
-          for (int s = 0; s < p.split; ++s)
+          for (int s = 0; s < p.split; ++s) {
+            const float* src = cl.map_shared_rank(part, s) + row;
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-              if (yoffk[k] >= 0) acc[k] += src[s * sl + colk[k]];
+              if (yoffk[k] >= 0) acc[k] += src[colk[k]];
+          }
 #pragma unroll
           for (int k = 0; k < 8; ++k)
             if (yoffk[k] >= 0) {
@@ -553,12 +537,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           for (int k = 0; k < 2; ++k)
 #pragma unroll
             for (int d = 0; d < 4; ++d) acc[k][d] = 0.f;
-          for (int s = 0; s < p.split; ++s)
+          for (int s = 0; s < p.split; ++s) {
+            const float* src = cl.map_shared_rank(part, s) + row;
 #pragma unroll
             for (int k = 0; k < 2; ++k)
               if (yoffk[k] >= 0)
 #pragma unroll
-                for (int d = 0; d < 4; ++d) acc[k][d] += src[s * sl + colk[k] + (d >> 1) * p.bcols + (d & 1)];
+                for (int d = 0; d < 4; ++d) acc[k][d] += src[colk[k] + (d >> 1) * p.bcols + (d & 1)];
+          }
 #pragma unroll
           for (int k = 0; k < 2; ++k)
             if (yoffk[k] >= 0) {
@@ -577,11 +563,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         }
       }
     }
-    if (issued) {
-      // the copies have landed before the CTA exits, also if the wait above gave up
-      for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&red_bar), 0u); ++k) {
-      }
-    }
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
   }
 
   tm_fence_before();
@@ -748,12 +731,12 @@ bool flat_pick(int N, int H, int W, int nch, int nfb, bool pool, const DeviceSta
 
 // The geometry pinned by timing for this shape, if any.
 bool pinned_geometry(const ppc::TcLayout& T, int N, int H, int W, int flags, const DeviceState& D, FlatGeo* out) {
-  const ppc::TcScratch* st = T.scratch;
+  const ppc::TcState* st = T.state;
   if (!st || st->R <= 0 || st->key[0] != N || st->key[1] != H || st->key[2] != W || st->key[3] != flags) return false;
   return flat_pick(N, H, W, T.nch, T.nfb, flags & PP_POOL2, D, st->R, st->S, out);
 }
 
-pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
+pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
                      const float* x, float* y, const float* skip, int N, int H, int W, int flags, cudaStream_t stream);
 
 }  // namespace
@@ -762,46 +745,21 @@ namespace ppc {
 
 pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N, int H,
                      int W, int flags, cudaStream_t stream) {
-  if (T.FB != FB || !T.scratch) return PP_ERR_UNSUPPORTED;
+  if (T.FB != FB) return PP_ERR_UNSUPPORTED;
   DeviceState* D = prepare();
   if (!D) return PP_ERR_CUDA;
   const bool pool = flags & PP_POOL2;
   FlatGeo G;
   if (!pinned_geometry(T, N, H, W, flags, *D, &G) && !flat_geometry(N, H, W, T.nch, T.nfb, pool, true, *D, &G))
     return PP_ERR_UNSUPPORTED;
-  if (G.split > 1) {
-    const size_t need = (size_t)G.ntiles * G.split * FB * G.ncols * sizeof(float);
-    if (T.scratch->bytes < need) {
-      // Grow the layer's split workspace, but never inside a stream capture:
-      // there the launch runs unsplit instead.
-      cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-      const bool capturing = cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone;
-      cudaGetLastError();
-      bool ok = false;
-      if (!capturing) {
-        if (T.scratch->p) cudaFree(T.scratch->p);
-        T.scratch->p = nullptr;
-        T.scratch->bytes = 0;
-        void* d = nullptr;
-        if (cudaMalloc(&d, need) == cudaSuccess) {
-          T.scratch->p = static_cast<float*>(d);
-          T.scratch->bytes = need;
-          ok = true;
-        } else {
-          cudaGetLastError();
-        }
-      }
-      if (!ok && !flat_geometry(N, H, W, T.nch, T.nfb, pool, false, *D, &G)) return PP_ERR_UNSUPPORTED;
-    }
-  }
-  return launch_geo(G, G.split > 1 ? T.scratch->p : nullptr, *D, T, M, x, y, skip, N, H, W, flags, stream);
+  return launch_geo(G, *D, T, M, x, y, skip, N, H, W, flags, stream);
 }
 
 }  // namespace ppc
 
 namespace {
 
-pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
+pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
                      const float* x, float* y, const float* skip, int N, int H, int W, int flags, cudaStream_t stream) {
   const DeviceState* D = &Dref;
   FlatParams p;
@@ -812,7 +770,6 @@ pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const
   p.perm = M.perm;
   p.bias = M.bias;
   p.status = T.status;
-  p.ws = ws;
   p.N = N;
   p.Ci = M.Ci;
   p.Co = M.Co;
@@ -878,13 +835,6 @@ pp_status launch_geo(const FlatGeo& G, float* ws, const DeviceState& Dref, const
   return PP_OK;
 }
 
-// Split workspace of the allocation-free entry point: one per device, shared
-// by every call on it.  Nothing in it needs to start at zero (each CTA writes
-// its whole partial tile before any CTA of its cluster reads it).
-constexpr size_t STATIC_WS_BYTES = (size_t)16 << 20;
-__device__ __align__(256) float g_static_ws[STATIC_WS_BYTES / sizeof(float)];
-float* g_static_ws_ptr[64] = {};
-
 }  // namespace
 
 namespace ppc {
@@ -903,42 +853,14 @@ int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, 
 }
 
 void tcf_pin(const TcLayout& T, int N, int H, int W, int flags, int R, int S) {
-  if (!T.scratch) return;
-  TcScratch* st = T.scratch;
+  if (!T.state) return;
+  TcState* st = T.state;
   st->key[0] = N;
   st->key[1] = H;
   st->key[2] = W;
   st->key[3] = flags;
   st->R = R;
   st->S = S;
-}
-
-pp_status tcf_launch_static(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
-                            int H, int W, int flags, cudaStream_t stream) {
-  if (T.FB != FB) return PP_ERR_UNSUPPORTED;
-  DeviceState* D = prepare();
-  if (!D) return PP_ERR_CUDA;
-  FlatGeo G;
-  if (!pinned_geometry(T, N, H, W, flags, *D, &G) &&
-      !flat_geometry(N, H, W, T.nch, T.nfb, flags & PP_POOL2, true, *D, &G))
-    return PP_ERR_UNSUPPORTED;
-  float* ws = nullptr;
-  if (G.split > 1) {
-    if ((size_t)G.ntiles * G.split * FB * G.ncols * sizeof(float) > STATIC_WS_BYTES) return PP_ERR_UNSUPPORTED;
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return PP_ERR_CUDA;
-    if (!g_static_ws_ptr[dev]) {
-      // once per device: the address of the static workspace
-      void* a = nullptr;
-      if (cudaGetSymbolAddress(&a, g_static_ws) != cudaSuccess || !a) {
-        cudaGetLastError();
-        return PP_ERR_CUDA;
-      }
-      g_static_ws_ptr[dev] = static_cast<float*>(a);
-    }
-    ws = g_static_ws_ptr[dev];
-  }
-  return launch_geo(G, ws, *D, T, M, x, y, skip, N, H, W, flags, stream);
 }
 
 }  // namespace ppc

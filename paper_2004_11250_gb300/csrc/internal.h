@@ -47,13 +47,9 @@ struct TmLayout {
   const uint4* blob = nullptr;
 };
 
-// Workspace of the split (cluster) launches of the flat tensor-core kernel:
-// one fp32 partial output tile per CTA.  Grown on demand outside stream capture.
-struct TcScratch {
-  float* p = nullptr;
-  size_t bytes = 0;
-  // Flat-kernel geometry chosen by timing (pp_layer_autotune) for one shape:
-  // rows per tile and split, used while (N, H, W, flags) match key.
+// Flat tensor-core kernel geometry chosen by timing (pp_layer_autotune) for one
+// shape: rows per tile R and split S, used while (N, H, W, flags) match key.
+struct TcState {
   int key[4] = {0, 0, 0, -1};
   int R = 0, S = 0;
 };
@@ -66,7 +62,7 @@ struct TcLayout {
   size_t dbytes = 0;
   const unsigned char* a = nullptr;
   int* status = nullptr;        // device word, nonzero after a timed-out wait
-  TcScratch* scratch = nullptr;  // owned; see tc_free
+  TcState* state = nullptr;  // owned; see tc_free
 };
 
 pp_status tc_prepare();
@@ -84,10 +80,6 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
 int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, int maxn);
 // Use geometry (R, S) for launches of this shape (R = 0: back to the model).
 void tcf_pin(const TcLayout& T, int N, int H, int W, int flags, int R, int S);
-// The same kernel with its split workspace in a fixed-size static device array
-// instead of the layer's (see pp_conv_forward_noalloc); never allocates.
-pp_status tcf_launch_static(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip,
-                            int N, int H, int W, int flags, cudaStream_t stream);
 
 // True when every pattern of the set is one of the ring patterns (centre plus
 // 3 consecutive neighbours); ring_of[p] receives its ring index.
