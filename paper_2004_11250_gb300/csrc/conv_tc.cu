@@ -206,6 +206,23 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           : "memory");
     };
     int raw_issued = 0, w_issued = 0;  // thread 0's counts of issued copies
+    // Weights of chunk gg into stage s (thread 0).
+    auto issue_w = [&](int gg, int s) {
+      const Tile T = tile_of(p, (int)blockIdx.x + (gg / p.nch) * (int)gridDim.x, G::R, TW);
+      const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + gg % p.nch) * G::W_BYTES;
+      mbar_arrive_expect_tx(su32(&wfull[s]), G::W_BYTES);
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              su32(smem + s * G::STAGE)),
+          "l"(src), "r"(G::W_BYTES), "r"(su32(&wfull[s]))
+          : "memory");
+    };
+    // The weights do not depend on the previous kernel in the stream: the first
+    // two chunks' copies start before waiting for it (programmatic dependent
+    // launch), everything that reads x comes after the wait.
+    if (tid == 0)
+      for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && G::SEP)
       for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + G::RAW_OFF + raw_issued * G::RAW);
     int g = 0;  // chunk sequence number of this CTA
@@ -223,14 +240,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         float4* hi = reinterpret_cast<float4*>(st + G::W_BYTES);
         float4* lo = reinterpret_cast<float4*>(st + G::W_BYTES + G::IN_BYTES);
         if (tid == 0) {
-          const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * G::W_BYTES;
-          mbar_arrive_expect_tx(su32(&wfull[s]), G::W_BYTES);
-          asm volatile(
-              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                  su32(st)),
-              "l"(src), "r"(G::W_BYTES), "r"(su32(&wfull[s]))
-              : "memory");
-          ++w_issued;
+          if (g >= 2) {
+            issue_w(g, s);
+            ++w_issued;
+          }
           if (p.use_tma && !G::SEP) {
             issue_raw(g, reinterpret_cast<unsigned char*>(lo));
             ++raw_issued;
@@ -381,6 +394,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         mma_commit(su32(&acc_full[b]));
       }
       // every MMA issued by this thread is complete before TMEM is released
+      // the next kernel in the stream may start its prologue (it waits for this
+      // grid to complete before it reads anything this grid writes)
+      asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
       mma_commit(su32(&done_bar));
       wait(&done_bar, 0u);
     }
@@ -589,6 +605,13 @@ cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
   cfg.blockDim = dim3(NTHREADS);
   cfg.dynamicSmemBytes = G::SMEM_ALLOC;
   cfg.stream = stream;
+  // programmatic dependent launch: the kernel waits (griddepcontrol.wait) for
+  // the previous one before touching its inputs and outputs
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB>, p, xmap);
 }
 

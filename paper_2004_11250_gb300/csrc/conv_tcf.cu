@@ -199,7 +199,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     };
     // With a ring of their own the boxes are copied two chunks ahead of use,
     // not only once the chunk's stage is free.
+    // Weights of chunk gg into stage s (thread 0).
+    auto issue_w = [&](int gg, int s) {
+      const Tile T = tile_of(p, tile_index(gg / nchm));
+      const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c_beg + gg % nchm) * W_BYTES;
+      mbar_arrive_expect_tx(su32(&wfull[s]), W_BYTES);
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              su32(smem + (size_t)s * p.stage)),
+          "l"(src), "r"(W_BYTES), "r"(su32(&wfull[s]))
+          : "memory");
+    };
     int g = 0, w_issued = 0, raw_issued = 0;
+    // The weights do not depend on the previous kernel in the stream: the first
+    // two chunks' copies start before waiting for it (programmatic dependent
+    // launch), everything that reads x comes after the wait.
+    if (tid == 0)
+      for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && p.sep)
       for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + p.raw_off + raw_issued * p.raw_slot);
     bool stop = false;  // identical in every loader thread (decided by group_any)
@@ -232,13 +249,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         float4* hi = reinterpret_cast<float4*>(st + W_BYTES);
         float4* lo = reinterpret_cast<float4*>(st + p.lo_off);
         if (tid == 0) {
-          const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
-          mbar_arrive_expect_tx(su32(&wfull[s]), W_BYTES);
-          asm volatile(
-              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(su32(st)),
-              "l"(src), "r"(W_BYTES), "r"(su32(&wfull[s]))
-              : "memory");
-          ++w_issued;
+          if (g >= 2) {
+            issue_w(g, s);
+            ++w_issued;
+          }
           if (p.use_tma && !p.sep) {
             issue_raw(g, reinterpret_cast<unsigned char*>(lo));  // lands in the lo operand, split in place below
             ++raw_issued;
@@ -331,6 +345,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         mma_commit(su32(&acc_full[b]));
       }
       // every MMA issued by this thread is complete before TMEM is released
+      // the next kernel in the stream may start its prologue (it waits for this
+      // grid to complete before it reads anything this grid writes)
+      asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
       mma_commit(su32(&done_bar));
       wait(&done_bar, 0u);
     }
@@ -810,18 +827,23 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
                       : 0;
   }
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
+  // programmatic dependent launch: the kernel waits (griddepcontrol.wait) for
+  // the previous one before touching its inputs and outputs
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
   cfg.blockDim = dim3(NTHREADS);
   cfg.dynamicSmemBytes = SMEM_ALLOC;
   cfg.stream = stream;
   cudaError_t e;
   if (G.split > 1) {
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = (unsigned)G.split;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = (unsigned)G.split;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
     cfg.gridDim = dim3((unsigned)(G.ntiles * G.split));
     e = cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true>, p, xmap);
   } else {
