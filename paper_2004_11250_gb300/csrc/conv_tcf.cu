@@ -65,7 +65,6 @@ constexpr int IN_MAX = 2 * PIX_MAX * 16;  // largest hi (or lo) operand of one c
 constexpr int SMEM_ALLOC = 231424;    // dynamic shared memory (static use stays below 1 KB)
 constexpr int SMEM_USE = SMEM_ALLOC - 1024;  // after aligning the base to 1024
 constexpr int ITEMS_MAX = (2 * PIX_MAX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
-constexpr int PF_AHEAD = 16;          // first chunks whose operands are prefetched into L2
 constexpr long WAIT_LIMIT = 1L << 22;
 constexpr int MAX_SPLIT = 16;
 static_assert(2 * (W_BYTES + 2 * IN_MAX) <= SMEM_USE, "shared memory plan");
@@ -354,24 +353,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
-    if (tid == (EPI_WARP0 + 7) * 32) {
-      // While the loaders start, one epilogue thread (idle until the first
-      // accumulators are ready) sends the weights and input boxes of the CTA's
-      // first chunks on their way into L2.
-      const int nchm = c_end - c_beg;
-      for (int gg = 0; gg < nmine * nchm && gg < PF_AHEAD; ++gg) {
-        const int i = gg / nchm, c = c_beg + gg % nchm;
-        const Tile T = tile_of(p, tile_index(i));
-        const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c) * W_BYTES;
-        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(W_BYTES) : "memory");
-        if (p.use_tma)
-          asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
-                           reinterpret_cast<uint64_t>(&xmap)),
-                       "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n)
-                       : "memory");
-      }
-    }
-    __syncwarp();
     const int q = warp & 3;                     // TMEM lane quadrant of this warp
     const int half = (warp - EPI_WARP0) >> 2;   // the two warps of a quadrant share the work
     const bool pool = p.flags & PP_POOL2;
