@@ -99,6 +99,103 @@ __device__ __forceinline__ Tile tile_of(const FlatParams& p, int t) {
   return T;
 }
 
+// Second phase of a cluster split: this CTA owns filters [m0, m0 + nm) of the
+// tile and sums, for each of them, the S partial tiles of the cluster (read in
+// rank order from each CTA's shared memory), then applies the epilogue.  Work
+// items are 4 adjacent accumulator columns of one filter (pooled: 2 rows x 4
+// columns, i.e. 2 pooled outputs), spread over all threads of the CTA; each
+// item issues its S 16-byte loads before it sums them.
+template <int S>
+__device__ __forceinline__ void split_reduce(const FlatParams& p, const Tile& T, int m0, int nm, float* part,
+                                             const int* o_s, const float* b_s, int tid) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  const float* src[S];
+#pragma unroll
+  for (int s = 0; s < S; ++s) src[s] = cl.map_shared_rank(part, s);
+  const int pst = p.ncols + 4;
+  const bool relu = p.flags & PP_RELU;
+  const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
+  auto sum = [&](int off) -> float4 {
+    float4 v[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) v[s] = *reinterpret_cast<const float4*>(src[s] + off);
+    float4 a = v[0];
+#pragma unroll
+    for (int s = 1; s < S; ++s) {
+      a.x += v[s].x;
+      a.y += v[s].y;
+      a.z += v[s].z;
+      a.w += v[s].w;
+    }
+    return a;
+  };
+  if (!(p.flags & PP_POOL2)) {
+    const int qw = (p.W + 3) >> 2, ipf = p.R * qw;
+    for (int it = tid; it < nm * ipf; it += NTHREADS) {
+      const int ml = it / ipf, rest = it - ml * ipf;
+      const int ro = rest / qw, cx = (rest - ro * qw) * 4;
+      const int row = T.r0 + ro, o = o_s[ml];
+      if (row >= p.H || o < 0) continue;
+      const float4 a = sum((m0 + ml) * pst + ro * p.bcols + cx);
+      const size_t yoff = (((size_t)T.n * p.Co + o) * p.H + row) * p.W + cx;
+      float v[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        v[k] += b_s[ml];
+        if (skip && cx + k < p.W) v[k] += __ldg(skip + yoff + k);
+        if (relu) v[k] = fmaxf(v[k], 0.f);
+      }
+      float* y = p.y + yoff;
+      if ((p.W & 3) == 0) {
+        *reinterpret_cast<float4*>(y) = make_float4(v[0], v[1], v[2], v[3]);
+      } else if ((p.W & 1) == 0) {
+        *reinterpret_cast<float2*>(y) = make_float2(v[0], v[1]);
+        if (cx + 2 < p.W) *reinterpret_cast<float2*>(y + 2) = make_float2(v[2], v[3]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if (cx + k < p.W) y[k] = v[k];
+      }
+    }
+  } else {
+    const int Ho = p.H / 2, Wo = p.W / 2;
+    const int qw = (Wo + 1) >> 1, ipf = (p.R / 2) * qw;
+    for (int it = tid; it < nm * ipf; it += NTHREADS) {
+      const int ml = it / ipf, rest = it - ml * ipf;
+      const int pr = rest / qw, pc = (rest - pr * qw) * 2;
+      const int orow = T.r0 / 2 + pr, o = o_s[ml];
+      if (orow >= Ho || o < 0) continue;
+      const int off = (m0 + ml) * pst + 2 * pr * p.bcols + 2 * pc;
+      const float4 a = sum(off), b = sum(off + p.bcols);
+      const size_t plane = (size_t)T.n * p.Co + o;
+      // window d of pooled output e: row 2 pr + (d >> 1), column 2 (pc + e) + (d & 1)
+      const float win[2][4] = {{a.x, a.y, b.x, b.y}, {a.z, a.w, b.z, b.w}};
+      float out[2];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        float mx = 0.f;
+#pragma unroll
+        for (int d = 0; d < 4; ++d) {
+          float v = win[e][d] + b_s[ml];
+          if (skip && pc + e < Wo)
+            v += __ldg(skip + (plane * p.H + 2 * orow + (d >> 1)) * p.W + 2 * (pc + e) + (d & 1));
+          if (relu) v = fmaxf(v, 0.f);
+          mx = d == 0 ? v : fmaxf(mx, v);
+        }
+        out[e] = mx;
+      }
+      float* y = p.y + (plane * Ho + orow) * Wo + pc;
+      if ((Wo & 1) == 0) {
+        *reinterpret_cast<float2*>(y) = make_float2(out[0], out[1]);
+      } else {
+        y[0] = out[0];
+        if (pc + 1 < Wo) y[1] = out[1];
+      }
+    }
+  }
+}
+
 template <bool SPLIT>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
   extern __shared__ unsigned char smem_raw[];
@@ -108,6 +205,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   __shared__ __align__(8) uint64_t full[2], wfull[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
+  __shared__ int o_s[FB / 2];    // split phase: original index of each owned filter (-1 beyond Co)
+  __shared__ float b_s[FB / 2];  // and its bias
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -457,108 +556,28 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // Every thread of every CTA of the cluster arrives at both cluster
     // barriers, also after an early stop, so they always complete.  The first
     // (release / acquire at cluster scope) orders every CTA's partial tile in
-    // its shared memory before the reads below; the second keeps each CTA's
-    // shared memory alive until the others have read it.
-    // This CTA finishes filters [m0, m1) of the tile with all its warps: warp w
-    // takes filters m0 + w, m0 + w + 17, ...; lane i of it holds the original
-    // index and bias of its i-th one, fetched now so the loads overlap the
-    // barrier wait.
-    namespace cg = cooperative_groups;
+    // its shared memory, and the filter table below, before the reads; the
+    // second keeps each CTA's shared memory alive until the others have read it.
+    // This CTA finishes filters [m0, m1) of the tile (at most FB / 2 of them);
+    // their original indices and biases are fetched now, so the loads overlap
+    // the barrier wait.
     const int tile = (int)blockIdx.x / p.split, rank = (int)blockIdx.x % p.split;
     const int m0 = rank * FB / p.split, m1 = (rank + 1) * FB / p.split, nm = m1 - m0;
-    int o_l = -1;
-    float b_l = 0.f;
-    {
-      const int ml = warp + (NTHREADS / 32) * lane;
-      const int jr = tile_of(p, tile).fb * FB + m0 + ml;
-      if (ml < nm && jr < p.Co) {
-        o_l = __ldg(p.perm + jr);
-        b_l = p.bias ? __ldg(p.bias + jr) : 0.f;
-      }
+    const Tile T = tile_of(p, tile);
+    if (tid < nm) {
+      const int jr = T.fb * FB + m0 + tid;
+      o_s[tid] = jr < p.Co ? __ldg(p.perm + jr) : -1;
+      b_s[tid] = (jr < p.Co && p.bias) ? __ldg(p.bias + jr) : 0.f;
     }
     __syncwarp();
     asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
     if (!abort_s) {
-      cg::cluster_group cl = cg::this_cluster();
-      const Tile T = tile_of(p, tile);
-      const bool pool = p.flags & PP_POOL2;
-      const bool relu = p.flags & PP_RELU;
-      const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
-      const int pst = p.ncols + 4;
       float* part = reinterpret_cast<float*>(smem);
-      // Each lane's output pixels are the same for every filter: lane + 32 k of
-      // the tile's R x W (pooled: R/2 x W/2) pixels, k < 8 (R * W <= 256).  Their
-      // accumulator columns and output offsets are computed once; each filter
-      // then issues all its loads of the S partials (rank order, read from the
-      // cluster's shared memories) before using them.
-      const int Ro = pool ? p.R / 2 : p.R, Wo = pool ? p.W / 2 : p.W;
-      const int Ho = pool ? p.H / 2 : p.H;
-      const int r0o = pool ? T.r0 / 2 : T.r0;
-      int colk[8], yoffk[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const int j = lane + 32 * k;
-        const int ro = j / Wo, cx = j - ro * Wo;
-        const bool ok = j < Ro * Wo && r0o + ro < Ho;
-        colk[k] = pool ? 2 * ro * p.bcols + 2 * cx : ro * p.bcols + cx;
-        yoffk[k] = ok ? (r0o + ro) * Wo + cx : -1;
-      }
-      for (int ml = warp, i = 0; ml < nm; ml += NTHREADS / 32, ++i) {
-        const int o = __shfl_sync(0xffffffffu, o_l, i);
-        const float bs = __shfl_sync(0xffffffffu, b_l, i);
-        if (o < 0) break;  // warp-uniform; later filters are beyond Co too
-        const size_t plane = (size_t)T.n * p.Co + o;
-        const int row = (m0 + ml) * pst;
-        float* yp = p.y + plane * (size_t)Ho * Wo;
-        const float* sp = skip ? skip + plane * (size_t)p.H * p.W : nullptr;
-        if (!pool) {
-          float acc[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) acc[k] = 0.f;
-          for (int s = 0; s < p.split; ++s) {
-            const float* src = cl.map_shared_rank(part, s) + row;
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-              if (yoffk[k] >= 0) acc[k] += src[colk[k]];
-          }
-#pragma unroll
-          for (int k = 0; k < 8; ++k)
-            if (yoffk[k] >= 0) {
-              float v = acc[k] + bs;
-              if (sp) v += __ldg(sp + yoffk[k]);
-              if (relu) v = fmaxf(v, 0.f);
-              yp[yoffk[k]] = v;
-            }
-        } else {
-          float acc[2][4];
-#pragma unroll
-          for (int k = 0; k < 2; ++k)
-#pragma unroll
-            for (int d = 0; d < 4; ++d) acc[k][d] = 0.f;
-          for (int s = 0; s < p.split; ++s) {
-            const float* src = cl.map_shared_rank(part, s) + row;
-#pragma unroll
-            for (int k = 0; k < 2; ++k)
-              if (yoffk[k] >= 0)
-#pragma unroll
-                for (int d = 0; d < 4; ++d) acc[k][d] += src[colk[k] + (d >> 1) * p.bcols + (d & 1)];
-          }
-#pragma unroll
-          for (int k = 0; k < 2; ++k)
-            if (yoffk[k] >= 0) {
-              // full-resolution position of the window's top-left pixel
-              const int po = yoffk[k] / Wo, pc = yoffk[k] - po * Wo;
-              float mx = 0.f;
-#pragma unroll
-              for (int d = 0; d < 4; ++d) {
-                float v = acc[k][d] + bs;
-                if (sp) v += __ldg(sp + (size_t)(2 * po + (d >> 1)) * p.W + 2 * pc + (d & 1));
-                if (relu) v = fmaxf(v, 0.f);
-                mx = d == 0 ? v : fmaxf(mx, v);
-              }
-              yp[yoffk[k]] = mx;
-            }
-        }
+      switch (p.split) {
+        case 2: split_reduce<2>(p, T, m0, nm, part, o_s, b_s, tid); break;
+        case 4: split_reduce<4>(p, T, m0, nm, part, o_s, b_s, tid); break;
+        case 8: split_reduce<8>(p, T, m0, nm, part, o_s, b_s, tid); break;
+        default: split_reduce<16>(p, T, m0, nm, part, o_s, b_s, tid); break;
       }
     }
     __syncwarp();

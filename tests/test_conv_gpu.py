@@ -160,22 +160,24 @@ FLAT_CASES = [
     (1, 48, 136, 6, 128),
     (4, 32, 256, 20, 20),
     (1, 8, 136, 3, 2),
+    (1, 64, 130, 13, 15),
 ]
 
 
 @pytest.mark.parametrize("case", FLAT_CASES)
-@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu", "skip_pool_relu"])
 def test_tensor_core_flat_kernel(pp, runner, oracle_mod, case, flags):
     """The flat tensor-core kernel (whole rows per MMA, cluster split for few tiles) against the oracle."""
     N, Ci, Co, H, W = case
-    if flags == "pool_relu" and (H % 2 or W % 2):
+    pool = "pool" in flags
+    if pool and (H % 2 or W % 2):
         pytest.skip("pool needs even sizes")
     rng = np.random.default_rng(11 * sum(case) + len(flags))
     L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.45, ring=sum(case) % 2 == 0)
     x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
-    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
-    g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=pp.PP_KERNEL_TC_FLAT)
-    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if "skip" in flags else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", pool, kernel=pp.PP_KERNEL_TC_FLAT)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", pool)
     check_within(g, y, s, f"flat tensor-core kernel {case} {flags}")
 
 
