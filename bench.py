@@ -410,8 +410,9 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--kernels", default="",
-                    help="comma list, one per op (tm, reg, tc, flat, or auto to keep the autotuned choice): pins "
-                         "each op's kernel after pp_net_finalize, e.g. to profile the selection of an earlier run")
+                    help="comma list, one per op (tm, reg, tc, flat, flat:R:S, or auto to keep the autotuned "
+                         "choice): pins each op's kernel (and for flat:R:S the flat kernel's rows per tile and "
+                         "split) after pp_net_finalize, e.g. to profile the selection of an earlier run")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     ws, rank, local = dist_setup(args)
@@ -439,9 +440,12 @@ def main():
         names = args.kernels.split(",")
         if len(names) != len(dn.layers):
             raise SystemExit(f"--kernels needs {len(dn.layers)} entries")
-        for L, k in zip(dn.layers, names):
+        for L, k, op, sh in zip(dn.layers, names, spec.ops, shapes):
             if k != "auto" and not L.dense:
-                pp.pp_layer_set_kernel(L.handle, ids[k])
+                pp.pp_layer_set_kernel(L.handle, ids[k.split(":")[0]])
+                if k.startswith("flat:"):
+                    R, S = (int(v) for v in k.split(":")[1:])
+                    pp.pp_layer_pin_flat_geometry(L.handle, sh["N"], sh["H"], sh["W"], runner.op_flags(op), R, S)
     x = torch.from_numpy(spec.x).cuda()
     y = torch.empty(dn.out_shape, device="cuda")
     torch.cuda.synchronize()
@@ -477,6 +481,14 @@ def main():
     from paper_2004_11250_gb300 import ppconv as pp
     kern = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "ppconv_kernel (dense)"
             for L in dn.layers]
+    # the flat kernel's tile geometry per op ("R:S", as --kernels flat:R:S takes it)
+    geo = []
+    for L, op, sh in zip(dn.layers, spec.ops, shapes):
+        g = None
+        if not L.dense and pp.pp_layer_kernel(L.handle) == pp.PP_KERNEL_TC_FLAT:
+            R, S = pp.pp_layer_flat_geometry(L.handle, sh["N"], sh["H"], sh["W"], runner.op_flags(op))
+            g = f"{R}:{S}" if R else "model"
+        geo.append(g)
     tc_ops = [k for k in pruned if kern[k] in ("ppconv_tc_kernel", "ppconv_tcf_kernel")]
     tensor = None
     if tc_ops:
@@ -539,6 +551,7 @@ def main():
                          "hbm_peak_gbs": hbm, "hbm_peak_source": hbm_src},
             "layer_roofline_frac": layer_fracs,
             "layer_kernels": kern,
+            "layer_flat_geometry": geo,
             "clocks": clk,
             "cpu_baseline": cpu,
             "configs": configs,

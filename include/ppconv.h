@@ -199,6 +199,25 @@ pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
  * Errors: PP_ERR_INVALID_ARG, PP_ERR_UNSUPPORTED, PP_ERR_CUDA, PP_ERR_OOM. */
 pp_status pp_layer_autotune(pp_layer* layer, int N, int H, int W, int flags, void* stream);
 
+/* Tile geometry of the flat tensor-core kernel (PP_KERNEL_TC_FLAT) for launches
+ * of shape (N, H, W, flags): R output rows per tile and a cluster split of the
+ * input-channel chunks over S CTAs.  pp_layer_flat_geometry reports the pinned
+ * pair (R = S = 0 when none is pinned for that shape: the kernel's cost model
+ * then decides).  pp_layer_pin_flat_geometry pins (R, S) for that shape, as
+ * pp_layer_autotune does with the pair it measured fastest; R = 0 unpins.  One
+ * shape is pinned per layer (a new pin replaces the old).  This lets a tuning
+ * result be stored and re-applied without timing again.  Host-only, no device
+ * work.  Errors: PP_ERR_INVALID_ARG; PP_ERR_UNSUPPORTED when the layer has no
+ * flat-kernel layout (fewer than 65 filters) or the kernel cannot run (R, S)
+ * for that shape (R rows of round_up(W + 2, 8) pixels must fit one MMA of at
+ * most 256 columns, R even when pooling; S a power of 2 up to 16, at most the
+ * number of 8-channel chunks, with tiles x S within the SM count and the
+ * cluster size launchable on this GPU).  Every geometry stays within the
+ * error bound; geometries with different splits group the channel sum
+ * differently, so their last bits may differ (each is deterministic). */
+pp_status pp_layer_flat_geometry(const pp_layer* layer, int N, int H, int W, int flags, int* R, int* S);
+pp_status pp_layer_pin_flat_geometry(pp_layer* layer, int N, int H, int W, int flags, int R, int S);
+
 /* Synchronous: *device_error = 0 unless a kernel of this layer gave up a
  * bounded wait (its output is then invalid); the word is cleared by the read. */
 pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);

@@ -792,6 +792,23 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
   return st;
 }
 
+extern "C" pp_status pp_layer_flat_geometry(const pp_layer* L, int N, int H, int W, int flags, int* R, int* S) {
+  if (!L || !R || !S || N < 1 || H < 1 || W < 1) return PP_ERR_INVALID_ARG;
+  *R = 0;
+  *S = 0;
+  if (L->tc_ok && L->tc.FB == 128) ppc::tcf_pinned(L->tc, N, H, W, flags, R, S);
+  return PP_OK;
+}
+
+extern "C" pp_status pp_layer_pin_flat_geometry(pp_layer* L, int N, int H, int W, int flags, int R, int S) {
+  if (!L || N < 1 || H < 1 || W < 1 || R < 0) return PP_ERR_INVALID_ARG;
+  if (flags & ~(PP_ADD_SKIP | PP_RELU | PP_POOL2)) return PP_ERR_INVALID_ARG;
+  if (!L->tc_ok || L->tc.FB != 128) return PP_ERR_UNSUPPORTED;
+  if (R > 0 && !ppc::tcf_can_run(L->tc, N, H, W, flags, R, S)) return PP_ERR_UNSUPPORTED;
+  ppc::tcf_pin(L->tc, N, H, W, flags, R, S);
+  return PP_OK;
+}
+
 extern "C" pp_status pp_layer_device_status(const pp_layer* L, int* device_error) {
   if (!L || !device_error) return PP_ERR_INVALID_ARG;
   *device_error = 0;

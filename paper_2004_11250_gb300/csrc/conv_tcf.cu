@@ -874,6 +874,20 @@ int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, 
   return n;
 }
 
+bool tcf_can_run(const TcLayout& T, int N, int H, int W, int flags, int R, int S) {
+  if (T.FB != FB) return false;
+  DeviceState* D = prepare();
+  FlatGeo G;
+  return D && flat_pick(N, H, W, T.nch, T.nfb, flags & PP_POOL2, *D, R, S, &G);
+}
+
+void tcf_pinned(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S) {
+  const TcState* st = T.state;
+  const bool hit = st && st->R > 0 && st->key[0] == N && st->key[1] == H && st->key[2] == W && st->key[3] == flags;
+  *R = hit ? st->R : 0;
+  *S = hit ? st->S : 0;
+}
+
 void tcf_pin(const TcLayout& T, int N, int H, int W, int flags, int R, int S) {
   if (!T.state) return;
   TcState* st = T.state;

@@ -80,6 +80,10 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
 int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, int maxn);
 // Use geometry (R, S) for launches of this shape (R = 0: back to the model).
 void tcf_pin(const TcLayout& T, int N, int H, int W, int flags, int R, int S);
+// True when the flat kernel can run geometry (R, S) for this shape.
+bool tcf_can_run(const TcLayout& T, int N, int H, int W, int flags, int R, int S);
+// The geometry pinned for this shape, or R = S = 0.
+void tcf_pinned(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S);
 
 // True when every pattern of the set is one of the ring patterns (centre plus
 // 3 consecutive neighbours); ring_of[p] receives its ring index.

@@ -64,6 +64,8 @@ _SIGS = {
     "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_device_status": ([_P, _P], _I),
     "pp_layer_autotune": ([_P, _I, _I, _I, _I, _P], _I),
+    "pp_layer_flat_geometry": ([_P, _I, _I, _I, _I, _P, _P], _I),
+    "pp_layer_pin_flat_geometry": ([_P, _I, _I, _I, _I, _I, _I], _I),
     "pp_layer_destroy": ([_P], None),
     "pp_dense_create": ([_P, _P, _I, _I, _P, _PP], _I),
     "pp_dense_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
@@ -228,6 +230,17 @@ def pp_layer_kernel(layer) -> int:
 
 def pp_layer_autotune(layer, N, H, W, flags, stream=None):
     _check(lib.pp_layer_autotune(layer, N, H, W, flags, _stream(stream)), "pp_layer_autotune")
+
+
+def pp_layer_flat_geometry(layer, N, H, W, flags):
+    """(R, S) pinned for the flat tensor-core kernel at this shape, (0, 0) if none."""
+    R, S = _I(), _I()
+    _check(lib.pp_layer_flat_geometry(layer, N, H, W, flags, ctypes.byref(R), ctypes.byref(S)), "pp_layer_flat_geometry")
+    return R.value, S.value
+
+
+def pp_layer_pin_flat_geometry(layer, N, H, W, flags, R, S):
+    _check(lib.pp_layer_pin_flat_geometry(layer, N, H, W, flags, R, S), "pp_layer_pin_flat_geometry")
 
 
 def pp_layer_device_status(layer) -> int:

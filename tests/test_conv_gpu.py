@@ -181,6 +181,43 @@ def test_tensor_core_flat_kernel(pp, runner, oracle_mod, case, flags):
     check_within(g, y, s, f"flat tensor-core kernel {case} {flags}")
 
 
+def test_flat_geometry_pin(pp, runner, oracle_mod):
+    """Every flat-kernel geometry the planner accepts for a shape gives results
+    within the bound; pins are reported back, rejected pairs raise, R = 0 unpins."""
+    N, Ci, Co, H, W = 1, 72, 130, 14, 14
+    rng = np.random.default_rng(5)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.45)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    y, s = oracle_layer_full(oracle_mod, L, x, None, True, True)
+    dl = runner.DeviceLayer(L)
+    flags = pp.PP_RELU | pp.PP_POOL2
+    try:
+        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC_FLAT)
+        assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, flags) == (0, 0)
+        accepted = []
+        for R in range(1, 17):
+            for S in (1, 2, 4, 8, 16):
+                try:
+                    pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, R, S)
+                except pp.PPError as e:
+                    assert e.code == pp.PP_ERR_UNSUPPORTED
+                    continue
+                assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, flags) == (R, S)
+                out = torch.full((N, Co, H // 2, W // 2), float("nan"), device="cuda")
+                dl.forward(dev(x), out, None, N, H, W, flags, torch.cuda.current_stream())
+                torch.cuda.synchronize()
+                check_within(out.cpu().numpy(), y, s, f"flat geometry R={R} S={S}")
+                accepted.append((R, S))
+        assert len(accepted) >= 3 and any(S > 1 for _, S in accepted), accepted
+        assert all(R % 2 == 0 for R, _ in accepted)  # pooling needs row pairs
+        # another shape's pin is not reported for this one; R = 0 unpins
+        assert pp.pp_layer_flat_geometry(dl.handle, N, H + 2, W, flags) == (0, 0)
+        pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, 0, 0)
+        assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, flags) == (0, 0)
+    finally:
+        dl.close()
+
+
 @pytest.mark.parametrize("shape", [(1, 136, 130, 28, 28), (6, 40, 200, 14, 14)])
 def test_tensor_core_flat_integer_bit_exact(pp, runner, oracle_mod, shape):
     """Integer weights and inputs: tf32 holds them exactly (lo parts are zero) and
