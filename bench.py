@@ -43,7 +43,8 @@ if ROOT not in sys.path:
 HBM_PEAK_GBS_FALLBACK = 6800.0
 BF16_PEAK_TFLOPS_FALLBACK = 1900.0
 TF32_PER_BF16 = 1.1 / 2.25  # nominal dense tensor rates
-KERNEL_NAMES = {1: "ppconv_tm_kernel", 2: "ppconv_kernel", 3: "ppconv_tc_kernel", 4: "ppconv_tcf_kernel"}
+KERNEL_NAMES = {1: "ppconv_tm_kernel", 2: "ppconv_kernel", 3: "ppconv_tc_kernel", 4: "ppconv_tcf_kernel",
+                5: "ppconv_direct_kernel"}
 SM_COUNT = 152
 FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
@@ -269,7 +270,7 @@ def kernel_source_hash():
     """sha256 over the conv kernel sources (a profile taken on other sources is stale)."""
     import hashlib
     h = hashlib.sha256()
-    for name in ("conv.cu", "conv_tm.cu", "conv_tc.cu", "conv_tcf.cu", "tc_ptx.cuh", "internal.h"):
+    for name in ("conv.cu", "conv_tm.cu", "conv_tc.cu", "conv_tcf.cu", "conv_direct.cu", "tc_ptx.cuh", "internal.h"):
         with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()
@@ -410,7 +411,7 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--kernels", default="",
-                    help="comma list, one per op (tm, reg, tc, flat, flat:R:S, or auto to keep the autotuned "
+                    help="comma list, one per op (tm, reg, tc, flat, flat:R:S, direct, or auto to keep the autotuned "
                          "choice): pins each op's kernel (and for flat:R:S the flat kernel's rows per tile and "
                          "split) after pp_net_finalize, e.g. to profile the selection of an earlier run")
     args = ap.parse_args()
@@ -436,7 +437,7 @@ def main():
     if args.kernels:
         from paper_2004_11250_gb300 import ppconv as pp
         ids = {"tm": pp.PP_KERNEL_TMEM, "reg": pp.PP_KERNEL_REGISTER, "tc": pp.PP_KERNEL_TC,
-               "flat": pp.PP_KERNEL_TC_FLAT}
+               "flat": pp.PP_KERNEL_TC_FLAT, "direct": pp.PP_KERNEL_DIRECT}
         names = args.kernels.split(",")
         if len(names) != len(dn.layers):
             raise SystemExit(f"--kernels needs {len(dn.layers)} entries")

@@ -178,6 +178,10 @@ pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* 
  *                       consecutive of its 8 neighbours).
  *   PP_KERNEL_REGISTER  FP32 FMA over kept taps, accumulators in registers;
  *                       any pattern set.
+ *   PP_KERNEL_DIRECT    FP32 FMA over all 9 taps of dense [Co][Ci][9] weights
+ *                       (zeros where pruned), one 2 x 2 pixel block and up to
+ *                       16 filters per thread; layers with at most 16 input
+ *                       or at most 16 output channels (first and last layers).
  * PP_KERNEL_AUTO picks by an estimate of each kernel's time for the layer's
  * density.  Setting a kernel the layer cannot run returns PP_ERR_UNSUPPORTED. */
 #define PP_KERNEL_AUTO 0
@@ -185,6 +189,7 @@ pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* 
 #define PP_KERNEL_REGISTER 2
 #define PP_KERNEL_TC 3
 #define PP_KERNEL_TC_FLAT 4
+#define PP_KERNEL_DIRECT 5
 pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
 /* The kernel that pp_conv_forward will run (one of the PP_KERNEL_ values above, not _AUTO). */
 pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
@@ -232,7 +237,9 @@ typedef struct pp_dense pp_dense;
 /* w [Co][Ci][9] and bias [Co] (or NULL) are host fp32; copied to the device. */
 pp_status pp_dense_create(const float* w, const float* bias, int Co, int Ci, void* stream, pp_dense** out);
 
-/* Same contract as pp_conv_forward, over all 9 taps of every kernel. */
+/* Same contract as pp_conv_forward, over all 9 taps of every kernel.  Layers
+ * with at most 16 input or at most 16 output channels run the direct FMA
+ * kernel (PP_KERNEL_DIRECT); others the register-accumulator kernel. */
 pp_status pp_dense_forward(const pp_dense* layer, const float* x, float* y, const float* skip, int N, int H, int W,
                            int flags, void* stream);
 

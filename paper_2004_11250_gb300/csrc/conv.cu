@@ -400,6 +400,7 @@ struct pp_layer {
   int auto_kernel = 2;
   ppc::TmLayout tm;
   ppc::TcLayout tc;
+  ppc::DirectLayout direct;  // built for layers with few input or output channels
   int G = 0, nch = 0;
   int cc = CC;  // input channels per stage
   int64_t nE = 0;
@@ -553,6 +554,7 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   if ((flags & PP_ADD_SKIP) && !skip) return PP_ERR_INVALID_ARG;
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   if (((uintptr_t)y & 15) || ((uintptr_t)x & 3)) return PP_ERR_INVALID_ARG;
+  if (L->kernel == PP_KERNEL_DIRECT) return ppc::direct_launch(L->direct, x, y, skip, N, H, W, flags, stream);
   if (L->kernel == PP_KERNEL_TMEM || L->kernel == PP_KERNEL_TC || L->kernel == PP_KERNEL_TC_FLAT) {
     ppc::LayerMeta M;
     M.Co = L->Co;
@@ -671,6 +673,17 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
     if (st == PP_OK) st = ppc::tc_build(&L->tc, pk, (cudaStream_t)stream);
     L->tc_ok = st == PP_OK;
   }
+  if (st == PP_OK && ppc::direct_applicable(pk->Co, pk->Ci)) {
+    // dense [Co][Ci][9] in the original filter order, zeros where pruned
+    std::vector<float> wd((size_t)pk->Co * pk->Ci * 9, 0.f);
+    for (int j = 0; j < pk->Co; ++j)
+      for (int32_t e = pk->kptr[j]; e < pk->kptr[j + 1]; ++e) {
+        const uint8_t* t = &pk->taps[4 * pk->kpat[e]];
+        for (int s = 0; s < 4; ++s)
+          wd[((size_t)pk->perm[j] * pk->Ci + pk->kidx[e]) * 9 + t[s]] = pk->kw[(size_t)e * 4 + s];
+      }
+    st = ppc::direct_build(&L->direct, wd.data(), bias, pk->Co, pk->Ci, (cudaStream_t)stream);
+  }
   if (st != PP_OK) {
     pp_layer_destroy(L);
     return st;
@@ -684,6 +697,9 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
   const double fma_cycles = 4.0 * nk / 32.0;
   L->auto_kernel = (L->tc_ok && tc_cycles < fma_cycles) ? (L->tc.FB == 128 ? PP_KERNEL_TC_FLAT : PP_KERNEL_TC)
                                                          : (L->tm_ok ? PP_KERNEL_TMEM : PP_KERNEL_REGISTER);
+  // layers with a handful of input channels (a network's first layer) run the
+  // direct kernel: the others cannot fill their tiles
+  if (L->direct.w && pk->Ci <= 4) L->auto_kernel = PP_KERNEL_DIRECT;
   L->kernel = L->auto_kernel;
   *out = L;
   return PP_OK;
@@ -706,6 +722,10 @@ extern "C" pp_status pp_layer_set_kernel(pp_layer* L, int kernel) {
       L->kernel = kernel;
       return PP_OK;
     case PP_KERNEL_REGISTER: L->kernel = kernel; return PP_OK;
+    case PP_KERNEL_DIRECT:
+      if (!L->direct.w) return PP_ERR_UNSUPPORTED;
+      L->kernel = kernel;
+      return PP_OK;
     default: return PP_ERR_INVALID_ARG;
   }
 }
@@ -734,6 +754,7 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
     for (int k = 0; k < n; ++k) cand.push_back({PP_KERNEL_TC_FLAT, R[k], S[k]});
   }
   if (L->tm_ok) cand.push_back({PP_KERNEL_TMEM, 0, 0});
+  if (L->direct.w) cand.push_back({PP_KERNEL_DIRECT, 0, 0});
   if (cand.empty()) cand.push_back({PP_KERNEL_REGISTER, 0, 0});
   if (cand.size() == 1) {
     L->kernel = cand[0].kernel;
@@ -822,7 +843,9 @@ extern "C" pp_status pp_layer_info(const pp_layer* L, int* Co, int* Ci, int64_t*
   if (!L) return PP_ERR_INVALID_ARG;
   if (Co) *Co = L->Co;
   if (Ci) *Ci = L->Ci;
-  if (device_bytes) *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes + L->tc.dbytes);
+  if (device_bytes)
+    *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes + L->tc.dbytes +
+                              (L->direct.w ? ((size_t)L->Co * L->Ci * 9 + (L->direct.bias ? L->Co : 0)) * 4 : 0));
   return PP_OK;
 }
 
@@ -854,6 +877,7 @@ extern "C" void pp_layer_destroy(pp_layer* L) {
   if (L->dmem) cudaFree(L->dmem);
   if (L->tm.dmem) cudaFree(L->tm.dmem);
   ppc::tc_free(&L->tc);
+  ppc::direct_free(&L->direct);
   delete L;
 }
 
@@ -888,8 +912,12 @@ extern "C" pp_status pp_dense_create(const float* w, const float* bias, int Co, 
   }
   // three entries per kernel: 5 channels per stage keep a warp's stage at <= EMAX entries
   pp_status st = build_layer(&D->base, Co, Ci, 5, per_filter, perm, bias, (cudaStream_t)stream);
+  if (st == PP_OK && ppc::direct_applicable(Co, Ci)) {
+    st = ppc::direct_build(&D->base.direct, w, bias, Co, Ci, (cudaStream_t)stream);
+    if (st == PP_OK) D->base.kernel = D->base.auto_kernel = PP_KERNEL_DIRECT;
+  }
   if (st != PP_OK) {
-    delete D;
+    pp_dense_destroy(D);
     return st;
   }
   *out = D;
@@ -912,5 +940,6 @@ extern "C" pp_status pp_dense_info(const pp_dense* D, int* Co, int* Ci) {
 extern "C" void pp_dense_destroy(pp_dense* D) {
   if (!D) return;
   if (D->base.dmem) cudaFree(D->base.dmem);
+  ppc::direct_free(&D->base.direct);
   delete D;
 }

@@ -85,6 +85,21 @@ bool tcf_can_run(const TcLayout& T, int N, int H, int W, int flags, int R, int S
 // The geometry pinned for this shape, or R = S = 0.
 void tcf_pinned(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S);
 
+// Direct FMA kernel for layers with few input or few output channels: dense
+// [Co][Ci][9] fp32 weights (zeros where pruned) and the bias, original order.
+constexpr int kDirectMaxSmall = 16;
+struct DirectLayout {
+  void* dmem = nullptr;
+  const float* w = nullptr;
+  const float* bias = nullptr;
+  int Co = 0, Ci = 0;
+};
+bool direct_applicable(int Co, int Ci);
+pp_status direct_build(DirectLayout* D, const float* w_dense, const float* bias, int Co, int Ci, cudaStream_t stream);
+pp_status direct_launch(const DirectLayout& D, const float* x, float* y, const float* skip, int N, int H, int W,
+                        int flags, cudaStream_t stream);
+void direct_free(DirectLayout* D);
+
 // True when every pattern of the set is one of the ring patterns (centre plus
 // 3 consecutive neighbours); ring_of[p] receives its ring index.
 bool tm_supports(const uint8_t* taps, int P, std::vector<int>& ring_of);

@@ -38,6 +38,7 @@ PP_KERNEL_TMEM = 1
 PP_KERNEL_REGISTER = 2
 PP_KERNEL_TC = 3
 PP_KERNEL_TC_FLAT = 4
+PP_KERNEL_DIRECT = 5
 
 PP_ADD_SKIP = 1
 PP_RELU = 2

@@ -323,6 +323,57 @@ def test_integer_layer_bit_exact(pp, runner, oracle_mod, ring):
     assert (g3.astype(np.float64) == y).all()
 
 
+DIRECT_CASES = [
+    # N, Ci, Co, H, W: first-layer and last-layer shapes, ragged tiles and filter blocks
+    (1, 3, 64, 37, 46),
+    (2, 1, 64, 33, 64),
+    (1, 16, 16, 32, 32),
+    (1, 64, 1, 40, 72),
+    (3, 2, 5, 17, 23),
+    (1, 5, 17, 64, 30),
+    (2, 16, 3, 8, 8),
+    (1, 4, 20, 1, 1),
+]
+
+
+@pytest.mark.parametrize("case", DIRECT_CASES)
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu", "skip_pool_relu"])
+def test_direct_kernel(pp, runner, oracle_mod, case, flags):
+    """The direct FMA kernel (dense 9-tap weights, few input or output channels) against the oracle."""
+    N, Ci, Co, H, W = case
+    pool = "pool" in flags
+    if pool and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(7 * sum(case) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.6, ring=sum(case) % 2 == 1)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if "skip" in flags else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", pool, kernel=pp.PP_KERNEL_DIRECT)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", pool)
+    check_within(g, y, s, f"direct kernel {case} {flags}")
+
+
+def test_direct_kernel_integer_bit_exact_and_selection(pp, runner, oracle_mod):
+    """Integer weights and inputs are summed exactly; a 3-channel first layer picks the direct
+    kernel by default, a wide layer cannot set it."""
+    rng = np.random.default_rng(31)
+    L = synth.integer_layer(rng, 16, 12, synth.seeded_patterns(rng, 8), 0.5)
+    x = rng.integers(-8, 9, (2, 12, 19, 27)).astype(np.float32)
+    g = run_layer(pp, runner, L, x, kernel=pp.PP_KERNEL_DIRECT)
+    y, _ = oracle_layer_full(oracle_mod, L, x)
+    assert (g.astype(np.float64) == y).all()
+    first = runner.DeviceLayer(synth.small_random_layer(rng, 64, 3, P=8, keep=1.0))
+    wide = runner.DeviceLayer(synth.small_random_layer(rng, 32, 32, P=8, keep=0.5))
+    try:
+        assert pp.pp_layer_kernel(first.handle) == pp.PP_KERNEL_DIRECT
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_layer_set_kernel(wide.handle, pp.PP_KERNEL_DIRECT)
+        assert e.value.code == pp.PP_ERR_UNSUPPORTED
+    finally:
+        first.close()
+        wide.close()
+
+
 def test_all_pruned_layer_gives_bias(pp, runner, oracle_mod):
     rng = np.random.default_rng(8)
     L = synth.small_random_layer(rng, 20, 10, P=8, keep=0.0)
