@@ -25,8 +25,9 @@
 namespace {
 
 constexpr int DT = 32;        // output tile edge
-constexpr int DTW = DT + 2;   // staged rows and columns (one-pixel halo)
-constexpr int DPITCH = 36;    // shared-memory row pitch in floats (16-byte multiple)
+constexpr int DTW = DT + 2;   // staged rows (one-pixel halo)
+constexpr int DCOLS = DT + 8; // staged columns: c0 - 4 .. c0 + 35 (16-byte aligned groups of 4)
+constexpr int DPITCH = DCOLS; // shared-memory row pitch in floats
 constexpr int DTHREADS = 256;
 
 struct DirectParams {
@@ -37,17 +38,24 @@ struct DirectParams {
   const float* bias;  // [Co] or null
   int N, Ci, Co, H, W, flags;
   int tiles_x, tiles_y;
+  int vec;  // x 16-byte aligned and W a multiple of 4: rows staged in 16-byte copies
 };
 
 __device__ __forceinline__ void cp_async4(float* dst, const float* src, bool valid) {
   const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(src), "r"(valid ? 4 : 0) : "memory");
 }
+__device__ __forceinline__ void cp_async16(float* dst, const float* src, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(valid ? 16 : 0) : "memory");
+}
 
 template <int CC, int FBD>
 __global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const DirectParams p) {
-  __shared__ __align__(16) float xs[2][CC][DTW][DPITCH];
-  __shared__ __align__(16) float ws[2][CC][FBD][12];  // 9 taps padded to 12
+  // two stages of [CC][DTW][DPITCH] input and [CC][FBD][12] weights (9 taps padded to 12)
+  extern __shared__ __align__(16) float dsm[];
+  auto xs = reinterpret_cast<float(*)[CC][DTW][DPITCH]>(dsm);
+  auto ws = reinterpret_cast<float(*)[CC][FBD][12]>(dsm + 2 * CC * DTW * DPITCH);
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   int t = (int)blockIdx.x;
   const int bx = t % p.tiles_x;
@@ -61,13 +69,25 @@ __global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const Direct
 
   // channels ch * CC .. of the input tile (zero outside the image and beyond
   // Ci) and their weights for this CTA's filters (zero beyond Co) into buffer b
+  // staged column j holds image column c0 - 4 + j
   auto stage = [&](int ch, int b) {
-    for (int e = tid; e < CC * DTW * DTW; e += DTHREADS) {
-      const int k = e / (DTW * DTW), rem = e - k * (DTW * DTW);
-      const int rr = rem / DTW, cc = rem - rr * DTW;
-      const int c = ch * CC + k, r = r0 - 1 + rr, col = c0 - 1 + cc;
-      const bool in = c < p.Ci && (unsigned)r < (unsigned)p.H && (unsigned)col < (unsigned)p.W;
-      cp_async4(&xs[b][k][rr][cc], in ? xb + ((size_t)c * p.H + r) * p.W + col : p.x, in);
+    if (p.vec) {
+      // rows of 16-byte groups: with W a multiple of 4 each group is wholly inside or outside the image
+      for (int e = tid; e < CC * DTW * (DCOLS / 4); e += DTHREADS) {
+        const int k = e / (DTW * (DCOLS / 4)), rem = e - k * (DTW * (DCOLS / 4));
+        const int rr = rem / (DCOLS / 4), g = rem - rr * (DCOLS / 4);
+        const int c = ch * CC + k, r = r0 - 1 + rr, col = c0 - 4 + 4 * g;
+        const bool in = c < p.Ci && (unsigned)r < (unsigned)p.H && (unsigned)col < (unsigned)p.W;
+        cp_async16(&xs[b][k][rr][4 * g], in ? xb + ((size_t)c * p.H + r) * p.W + col : p.x, in);
+      }
+    } else {
+      for (int e = tid; e < CC * DTW * DTW; e += DTHREADS) {
+        const int k = e / (DTW * DTW), rem = e - k * (DTW * DTW);
+        const int rr = rem / DTW, cc = rem - rr * DTW;
+        const int c = ch * CC + k, r = r0 - 1 + rr, col = c0 - 1 + cc;
+        const bool in = c < p.Ci && (unsigned)r < (unsigned)p.H && (unsigned)col < (unsigned)p.W;
+        cp_async4(&xs[b][k][rr][cc + 3], in ? xb + ((size_t)c * p.H + r) * p.W + col : p.x, in);
+      }
     }
     for (int e = tid; e < CC * FBD * 9; e += DTHREADS) {
       const int k = e / (FBD * 9), rem = e - k * (FBD * 9);
@@ -97,17 +117,13 @@ __global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const Direct
     __syncthreads();
 #pragma unroll
     for (int k = 0; k < CC; ++k) {
-      // the thread's 4 x 4 input window: staged rows 2 ty .. 2 ty + 3, columns 2 tx .. 2 tx + 3
+      // the thread's 4 x 4 input window: staged rows 2 ty .. 2 ty + 3, image
+      // columns c0 + 2 tx - 1 .. c0 + 2 tx + 2 (staged 2 tx + 3 .. 2 tx + 6)
       float xv[4][4];
 #pragma unroll
-      for (int a = 0; a < 4; ++a) {
-        const float2 u = *reinterpret_cast<const float2*>(&xs[b][k][2 * ty + a][2 * tx]);
-        const float2 v = *reinterpret_cast<const float2*>(&xs[b][k][2 * ty + a][2 * tx + 2]);
-        xv[a][0] = u.x;
-        xv[a][1] = u.y;
-        xv[a][2] = v.x;
-        xv[a][3] = v.y;
-      }
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) xv[a][q] = xs[b][k][2 * ty + a][2 * tx + 3 + q];
 #pragma unroll
       for (int o = 0; o < FBD; ++o) {
         const float4 w0 = *reinterpret_cast<const float4*>(&ws[b][k][o][0]);
@@ -166,16 +182,31 @@ __global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const Direct
   }
 }
 
+template <int CC, int FBD>
+cudaError_t launch_one(const DirectParams& p, dim3 grid, cudaStream_t stream) {
+  constexpr int bytes = 2 * (CC * DTW * DPITCH + CC * FBD * 12) * 4;
+  static bool attr_set[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!attr_set[dev]) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(ppconv_direct_kernel<CC, FBD>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  ppconv_direct_kernel<CC, FBD><<<grid, DTHREADS, bytes, stream>>>(p);
+  return cudaGetLastError();
+}
+
 template <int CC>
 cudaError_t launch_cc(const DirectParams& p, int fbd, dim3 grid, cudaStream_t stream) {
   switch (fbd) {
-    case 1: ppconv_direct_kernel<CC, 1><<<grid, DTHREADS, 0, stream>>>(p); break;
-    case 2: ppconv_direct_kernel<CC, 2><<<grid, DTHREADS, 0, stream>>>(p); break;
-    case 4: ppconv_direct_kernel<CC, 4><<<grid, DTHREADS, 0, stream>>>(p); break;
-    case 8: ppconv_direct_kernel<CC, 8><<<grid, DTHREADS, 0, stream>>>(p); break;
-    default: ppconv_direct_kernel<CC, 16><<<grid, DTHREADS, 0, stream>>>(p); break;
+    case 1: return launch_one<CC, 1>(p, grid, stream);
+    case 2: return launch_one<CC, 2>(p, grid, stream);
+    case 4: return launch_one<CC, 4>(p, grid, stream);
+    case 8: return launch_one<CC, 8>(p, grid, stream);
+    default: return launch_one<CC, 16>(p, grid, stream);
   }
-  return cudaGetLastError();
 }
 
 int sm_count() {
@@ -238,6 +269,7 @@ pp_status direct_launch(const DirectLayout& D, const float* x, float* y, const f
   p.flags = flags;
   p.tiles_x = (W + DT - 1) / DT;
   p.tiles_y = (H + DT - 1) / DT;
+  p.vec = (W & 3) == 0 && ((uintptr_t)x & 15) == 0;
   // filters per CTA: up to 16, fewer when the layer has too few tiles to give
   // every SM a few CTAs (the input tile is then staged once per filter block)
   const int64_t nt = (int64_t)N * p.tiles_x * p.tiles_y;

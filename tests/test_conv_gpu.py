@@ -353,6 +353,28 @@ def test_direct_kernel(pp, runner, oracle_mod, case, flags):
     check_within(g, y, s, f"direct kernel {case} {flags}")
 
 
+def test_direct_kernel_input_only_4_byte_aligned(pp, runner, oracle_mod):
+    """An input that starts 4 bytes past a 16-byte boundary takes the 4-byte copy path (same results)."""
+    N, Ci, Co, H, W = 1, 3, 24, 20, 36
+    rng = np.random.default_rng(41)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.8)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    dl = runner.DeviceLayer(L)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_DIRECT)
+        buf = torch.zeros(x.size + 1, device="cuda")
+        xs = buf[1:].view(N, Ci, H, W)
+        xs.copy_(torch.from_numpy(x))
+        assert xs.data_ptr() % 16 == 4
+        out = torch.full((N, Co, H, W), float("nan"), device="cuda")
+        dl.forward(xs, out, None, N, H, W, pp.PP_RELU, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        y, s = oracle_layer_full(oracle_mod, L, x, None, True, False)
+        check_within(out.cpu().numpy(), y, s, "direct kernel, 4-byte aligned input")
+    finally:
+        dl.close()
+
+
 def test_direct_kernel_integer_bit_exact_and_selection(pp, runner, oracle_mod):
     """Integer weights and inputs are summed exactly; a 3-channel first layer picks the direct
     kernel by default, a wide layer cannot set it."""
