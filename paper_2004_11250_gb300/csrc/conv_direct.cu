@@ -283,7 +283,8 @@ pp_status direct_launch(const DirectLayout& D, const float* x, float* y, const f
     case 1: e = launch_cc<1>(p, fbd, grid, stream); break;
     case 2: e = launch_cc<2>(p, fbd, grid, stream); break;
     case 3: e = launch_cc<3>(p, fbd, grid, stream); break;
-    default: e = launch_cc<4>(p, fbd, grid, stream); break;
+    case 4: e = launch_cc<4>(p, fbd, grid, stream); break;
+    default: e = launch_cc<8>(p, fbd, grid, stream); break;  // fewer, larger copy steps
   }
   if (e != cudaSuccess) return PP_ERR_CUDA;
   return PP_OK;
