@@ -105,6 +105,9 @@ __global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const Direct
 #pragma unroll
     for (int q = 0; q < 4; ++q) acc[o][q] = 0.f;
 
+  // programmatic dependent launch: nothing of the previous kernel in the
+  // stream is read or overwritten before this wait
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   stage(0, 0);
   for (int ch = 0; ch < nchunks; ++ch) {
     const int b = ch & 1;
@@ -144,6 +147,8 @@ __global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const Direct
     __syncthreads();  // buffer b is restaged by the next iteration's copy
   }
 
+  // the next kernel may start its prologue (it waits for this grid to finish)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const bool relu = p.flags & PP_RELU, pool = p.flags & PP_POOL2;
   const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
   const int r = r0 + 2 * ty, c = c0 + 2 * tx;
@@ -194,8 +199,17 @@ cudaError_t launch_one(const DirectParams& p, dim3 grid, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  ppconv_direct_kernel<CC, FBD><<<grid, DTHREADS, bytes, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(DTHREADS);
+  cfg.dynamicSmemBytes = bytes;
+  cfg.stream = stream;
+  return cudaLaunchKernelEx(&cfg, ppconv_direct_kernel<CC, FBD>, p);
 }
 
 template <int CC>
