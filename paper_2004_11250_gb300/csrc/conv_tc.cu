@@ -67,7 +67,10 @@ constexpr long WAIT_LIMIT = 1L << 22;  // mbarrier polls before a wait gives up
 // Orientation of the GEMM on the tensor core.
 //   ORI_FP: M = 128 filters, N = TW pixels of one output row (narrow maps)
 //   ORI_PF: M = 128 pixels of one output row, N = FB filters (wide maps)
-enum { ORI_FP = 0, ORI_PF = 1 };
+//   ORI_PFR: pixel-major with whole rows flattened: M = 128 staged pixels =
+//     128 / TW rows of TW >= W + 2 columns (TW = 16, 32 or 64; the columns
+//     past W are computed and dropped), for narrow maps of 64-filter layers
+enum { ORI_FP = 0, ORI_PF = 1, ORI_PFR = 2 };
 
 struct TcParams {
   const float* x;
@@ -88,20 +91,28 @@ struct TcParams {
 // per block, R row segments per tile (one accumulator column range each).
 template <int ORI, int TW, int FB>
 struct Geo {
-  static_assert(ORI == ORI_FP ? FB == 128 : TW == 128, "orientation needs a 128-row M side");
+  static_assert(ORI == ORI_FP ? FB == 128 : (ORI == ORI_PF ? TW == 128 : (128 % TW == 0 && FB == 64)),
+                "orientation needs a 128-row M side");
   // MRG (pixel-major): the hi and lo weight tiles of a tap are one 2 FB-wide B
   // operand, so x_hi * [w_hi | w_lo] is one N = 2 FB MMA (the lo part lands in
   // accumulator columns FB .. 2 FB - 1 and the epilogue adds the two halves);
   // x_lo * w_hi is an N = FB MMA.  Two MMAs instead of three read the pixel
   // tile twice instead of three times.
-  static constexpr bool MRG = ORI == ORI_PF;
+  static constexpr bool MRG = ORI != ORI_FP;
   static constexpr int SEGC = ORI == ORI_FP ? TW : (MRG ? 2 * FB : FB);  // accumulator columns per row segment
-  static constexpr int R = NCOL / SEGC;                   // row segments per tile
-  static constexpr int BROWS = R + 2, BCOLS = TW + 2;
+  static constexpr int NSEG = NCOL / SEGC;                // MMA row segments per tile
+  static constexpr int RSEG = ORI == ORI_PFR ? 128 / TW : 1;  // output rows per segment
+  static constexpr int R = NSEG * RSEG;                   // output rows per tile
+  static constexpr int BROWS = R + 2, BCOLS = ORI == ORI_PFR ? TW : TW + 2;
   static constexpr int NPIX = BROWS * BCOLS;              // staged input pixels
-  static constexpr int IN_HALF = NPIX * 16;               // one K half (4 channels) of hi or lo
+  // flattened rows: the last segment's operand for the (2, 2) tap runs 2
+  // pixels past the staged tile (junk columns only); 16 pixels of slack
+  static constexpr int NPIXA = ORI == ORI_PFR ? NPIX + 16 : NPIX;
+  static constexpr int IN_HALF = NPIXA * 16;              // one K half (4 channels) of hi or lo
   static constexpr int IN_BYTES = 2 * IN_HALF;            // hi or lo, 8 channels
-  static constexpr int RAW_W = TW + 8;                    // tensor-map box width: columns c0-4 .. c0+TW+3
+  // tensor-map box width: columns c0-4 .. (staged column bc is box column bc + 3),
+  // a multiple of 4 so each box row is whole 16-byte units
+  static constexpr int RAW_W = (BCOLS + 3 + 3) / 4 * 4;
   static constexpr int RAW = KC * BROWS * RAW_W * 4;      // box [8 channels][BROWS][RAW_W], landed in the lo area
   static constexpr int LO_BYTES = IN_BYTES > RAW ? IN_BYTES : RAW;
   static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo
@@ -286,8 +297,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
               h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
               h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
-              hi[it] = h;
-              lo[it] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+              const int dst = it + (it >= G::NPIX ? G::NPIXA - G::NPIX : 0);  // K halves NPIXA apart
+              hi[dst] = h;
+              lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
             }
           }
         } else {
@@ -318,8 +330,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
                 h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
                 h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
                 h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
-                hi[it] = h;
-                lo[it] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+                const int dst = it + (it >= G::NPIX ? G::NPIXA - G::NPIX : 0);
+                hi[dst] = h;
+                lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
               }
             }
           }
@@ -369,9 +382,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             const int dy = t / 3, dx = t % 3;
             const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * G::W_TILE / 16);
             const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows: FB rows of 16 bytes
-#pragma unroll(G::R <= 8 ? G::R : 4)
-            for (int rr = 0; rr < G::R; ++rr) {
-              const uint64_t off = (uint64_t)((rr + dy) * G::BCOLS + dx);  // pixels of 16 bytes
+#pragma unroll(G::NSEG <= 8 ? G::NSEG : 4)
+            for (int rr = 0; rr < G::NSEG; ++rr) {
+              const uint64_t off = (uint64_t)((rr * G::RSEG + dy) * G::BCOLS + dx);  // pixels of 16 bytes
               const uint64_t xh = xh0 + off, xl = xl0 + off;
               const uint32_t d = dbase + (uint32_t)(rr * G::SEGC);
               if (ORI == ORI_FP) {
@@ -483,14 +496,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           pm[k] = jr < p.Co ? __ldg(p.perm + jr) : -1;
           bv[k] = (jr < p.Co && p.bias) ? __ldg(p.bias + jr) : 0.f;
         }
-        const int col = T.c0 + 32 * q + lane;
+        // flattened rows (ORI_PFR): lane j of a segment is row j / TW, column j % TW of it
+        const int jl = 32 * q + lane;
+        const int rsub = ORI == ORI_PFR ? jl / TW : 0;
+        const int col = ORI == ORI_PFR ? jl % TW : T.c0 + jl;
         const int Ho = p.H / 2, Wo = p.W / 2;
         const int HW = p.H * p.W, HWo = Ho * Wo;
         const size_t nco = (size_t)T.n * p.Co;
         float* ybase = p.y + nco * (size_t)(pool ? HWo : HW);
         const float* sbase = (p.flags & PP_ADD_SKIP) ? p.skip + nco * (size_t)HW : nullptr;
-        for (int rr = 0; rr < G::R; rr += (pool ? 2 : 1)) {
-          const int row = T.r0 + rr;
+        for (int rr = 0; rr < G::NSEG; rr += (pool ? 2 : 1)) {
+          const int row = T.r0 + rr * G::RSEG + rsub;
           const bool in0 = row < p.H && col < p.W;
           const int roff = row * p.W + col;
           const int poff = (row >> 1) * Wo + (col >> 1);
@@ -565,6 +581,9 @@ cudaError_t prepare() {
   if ((e = set_attr<ORI_FP, 128, 128>()) != cudaSuccess) return e;
   if ((e = set_attr<ORI_PF, 128, 64>()) != cudaSuccess) return e;
   if ((e = set_attr<ORI_PF, 128, 128>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_PFR, 16, 64>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_PFR, 32, 64>()) != cudaSuccess) return e;
+  if ((e = set_attr<ORI_PFR, 64, 64>()) != cudaSuccess) return e;
   if (dev < 64) g_done[dev] = true;
   return cudaSuccess;
 }
@@ -706,7 +725,11 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
 void tc_geometry(const TcLayout& T, int W, bool pool, int* ori, int* tw) {
   // a pixel-major tile with 128 filters holds one output row (its accumulator
   // row segment is 2 x 128 columns wide), and pooling needs row pairs
-  if ((T.FB == 64 || W >= 96) && !(T.FB == 128 && pool)) {
+  if (T.FB == 64 && !pool && W + 2 <= 64) {
+    // narrow map, 64 filters: whole rows flattened into the 128-pixel M side
+    *ori = ORI_PFR;
+    *tw = W + 2 <= 16 ? 16 : W + 2 <= 32 ? 32 : 64;
+  } else if ((T.FB == 64 || W >= 96) && !(T.FB == 128 && pool)) {
     *ori = ORI_PF;
     *tw = 128;
   } else {
@@ -741,6 +764,9 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
   cudaError_t e;
   if (ori == ORI_PF)
     e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, g_sms) : launch<ORI_PF, 128, 128>(p, stream, g_sms);
+  else if (ori == ORI_PFR)
+    e = tw == 16 ? launch<ORI_PFR, 16, 64>(p, stream, g_sms)
+                 : tw == 32 ? launch<ORI_PFR, 32, 64>(p, stream, g_sms) : launch<ORI_PFR, 64, 64>(p, stream, g_sms);
   else if (tw == 16)
     e = launch<ORI_FP, 16, 128>(p, stream, g_sms);
   else if (tw == 32)

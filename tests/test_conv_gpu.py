@@ -164,6 +164,31 @@ FLAT_CASES = [
 ]
 
 
+PFR_CASES = [
+    # N, Ci, Co, H, W: 64-filter layers on maps at most 62 wide run the row-tiled
+    # kernel with whole rows flattened into the 128-pixel M side (16/32/64-pixel pitch)
+    (1, 64, 64, 56, 56),
+    (2, 24, 40, 20, 14),
+    (1, 16, 64, 33, 30),
+    (3, 40, 33, 9, 5),
+    (1, 72, 64, 23, 62),
+]
+
+
+@pytest.mark.parametrize("case", PFR_CASES)
+@pytest.mark.parametrize("flags", ["none", "skip_relu"])
+def test_tensor_core_flattened_rows(pp, runner, oracle_mod, case, flags):
+    """Row-tiled tensor-core kernel, pixel-major with flattened rows, against the oracle."""
+    N, Ci, Co, H, W = case
+    rng = np.random.default_rng(13 * sum(case) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.4)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", False, kernel=pp.PP_KERNEL_TC)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", False)
+    check_within(g, y, s, f"flattened-row tensor-core kernel {case} {flags}")
+
+
 @pytest.mark.parametrize("case", FLAT_CASES)
 @pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu", "skip_pool_relu"])
 def test_tensor_core_flat_kernel(pp, runner, oracle_mod, case, flags):
