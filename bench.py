@@ -352,6 +352,22 @@ def dist_setup(args):
     return ws, rank, local
 
 
+def max_over_ranks(t_ms, ws, device):
+    """The slowest rank's time (every rank gets it); a collective only when ws > 1."""
+    if ws == 1:
+        return float(t_ms)
+    import torch
+    t = torch.tensor([float(t_ms)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(ws, flops_frame, steps, t_total_ms):
+    """Whole-job throughput in GFLOP/s: every rank ran `steps` frames of `flops_frame` surviving FLOPs
+    (replicas; weak scaling), timed by the slowest rank."""
+    return ws * flops_frame * steps / (t_total_ms * 1e-3) / 1e9
+
+
 def run_reference(args, ws, rank):
     if rank != 0:
         return
@@ -460,14 +476,11 @@ def main():
         ts = time_net(dn, x, y, args.steps, args.warmup, flush, stream)
         torch.cuda.synchronize()
         clk = clocks.stop()
-    t_total_ms = sum(ts)
+    t_total_ms = max_over_ranks(sum(ts), ws, "cuda")
     if ws > 1:
-        t = torch.tensor([t_total_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        t_total_ms = float(t.item())
         torch.distributed.barrier()
     ms_per_step = t_total_ms / args.steps
-    value = ws * flops_frame * args.steps / (t_total_ms * 1e-3) / 1e9
+    value = job_value(ws, flops_frame, args.steps, t_total_ms)
 
     # per-op kernel durations (same stream, L2 flushed before each launch) -> roofline of the pruned conv
     acts = dn.run_layerwise(x, stream)
