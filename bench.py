@@ -241,9 +241,10 @@ def time_ops(dn, acts, steps, flush, stream):
     return res
 
 
-def traffic_from_profile(kernel_hash: str):
-    """Per-launch DRAM bytes of the pruned-conv kernel from the committed ncu summary, if that summary
-    was taken on the current kernel source."""
+def traffic_from_profile(kernel_hash: str, kernel: str = None):
+    """Per-launch DRAM bytes (read + write) from the committed ncu summary of the VGG-16 frame, of one
+    kernel (average over its launches in the frame) or of all the frame's convs, if that summary was
+    taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", "ppconv_vgg16_dram_traffic.txt")
     try:
         kv = {}
@@ -253,7 +254,8 @@ def traffic_from_profile(kernel_hash: str):
                 kv[k.strip()] = v.strip()
         if kv.get("kernel_source_sha256") != kernel_hash:
             return None
-        return float(kv["dram_bytes_per_launch_avg"])
+        key = f"dram_bytes_per_launch_avg[{kernel}]" if kernel else "dram_bytes_per_launch_avg"
+        return float(kv[key])
     except Exception:
         return None
 
@@ -490,7 +492,7 @@ def main():
     pruned = [k for k, s in enumerate(shapes) if s["pruned"]]
     kf = sum(shapes[k]["flops"] for k in pruned)
     kt = sum(op_ms[k] for k in pruned) * 1e-3
-    achieved = kf / kt / 1e12
+    achieved_all = kf / kt / 1e12
     # which kernel each op runs (autotuned by pp_net_finalize) and the tensor-pipe view
     from paper_2004_11250_gb300 import ppconv as pp
     kern = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "ppconv_kernel (dense)"
@@ -515,7 +517,16 @@ def main():
         tensor = {"bound": "tensor", "ops": len(tc_ops), "achieved": round(tf / tt / 1e12, 2), "peak": round(tpk, 1),
                   "unit": "TFLOP/s (tf32, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
                   "peak_source": f"{bsrc} bf16 {bpk} TFLOP/s x nominal tf32/bf16 {TF32_PER_BF16:.3f}"}
-    traffic = traffic_from_profile(kernel_source_hash())
+    # the dominant kernel (most device time over the pruned ops): its surviving FLOPs per launch over
+    # its mean launch duration, against the FP32 roofline of the method
+    by_kern = {}
+    for k in pruned:
+        f, t = by_kern.get(kern[k], (0.0, 0.0))
+        by_kern[kern[k]] = (f + shapes[k]["flops"], t + op_ms[k] * 1e-3)
+    dom = max(by_kern, key=lambda n: by_kern[n][1])
+    dom_ops = [k for k in pruned if kern[k] == dom]
+    achieved = by_kern[dom][0] / by_kern[dom][1] / 1e12
+    traffic = traffic_from_profile(kernel_source_hash(), dom)
     layer_fracs = [round(roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3), 3) for s, t in zip(shapes, op_ms)]
 
     # end to end through the public API with host buffers
@@ -559,7 +570,12 @@ def main():
             "gpu_launches": len(spec.ops) * args.steps,
             "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
                          "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
-                         "kernel": "all pruned ops of a step: " + ", ".join(sorted(set(kern[k] for k in pruned))),
+                         "kernel": f"{dom} ({len(dom_ops)} of the {len(pruned)} pruned convs, "
+                                   f"{100 * by_kern[dom][1] / kt:.0f}% of their device time)",
+                         "all_pruned_ops": {"achieved": round(achieved_all, 3),
+                                            "frac": round(achieved_all / FP32_PEAK_TFLOPS, 4),
+                                            "traffic": traffic_from_profile(kernel_source_hash()),
+                                            "kernels": sorted(by_kern)},
                          "tensor": tensor,
                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
                          "hbm_peak_gbs": hbm, "hbm_peak_source": hbm_src},
