@@ -112,6 +112,19 @@ pp_status pp_unpack_layer(const pp_packed* pk, float* w_out, uint8_t* mask_out);
 
 void pp_packed_destroy(pp_packed* pk);
 
+/* Fold an inference batch normalisation that follows the convolution into its
+ * weights and bias (Section 3: convolution fused with the layers after it), in
+ * place on host arrays before packing: w [Co][Ci][9] becomes w * g[o] and
+ * bias [Co] becomes (bias - mean) * g[o] + beta, with g[o] = gamma[o] /
+ * sqrt(var[o] + eps) evaluated in double and each result rounded once to fp32.
+ * One factor per filter keeps every zero weight zero, so a pattern-pruned and
+ * connectivity-pruned layer stays one (same masks, same pattern ids).  bias
+ * must be an array of Co (zeros for a convolution without bias).  Host only,
+ * synchronous.  Errors: PP_ERR_INVALID_ARG (null pointer, Co or Ci < 1, eps
+ * negative or NaN, var[o] + eps not positive). */
+pp_status pp_fold_batchnorm(float* w, float* bias, const float* gamma, const float* beta, const float* mean,
+                            const float* var, float eps, int Co, int Ci);
+
 /* ------------------------------------------------------------------------
  * Device layer: the pruned convolution on the GPU (Sections 2-3).
  * ------------------------------------------------------------------------ */

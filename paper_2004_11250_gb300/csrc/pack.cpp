@@ -10,6 +10,7 @@
 // reading (documented at pp_pack_layer in ppconv.h): the paper names the goal
 // (load balance, regular access) but not the key.
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <new>
 #include <numeric>
@@ -198,6 +199,23 @@ extern "C" pp_status pp_unpack_layer(const pp_packed* pk, float* w_out, uint8_t*
 }
 
 extern "C" void pp_packed_destroy(pp_packed* pk) { delete pk; }
+
+extern "C" pp_status pp_fold_batchnorm(float* w, float* bias, const float* gamma, const float* beta,
+                                       const float* mean, const float* var, float eps, int Co, int Ci) {
+  if (!w || !bias || !gamma || !beta || !mean || !var || Co < 1 || Ci < 1 || !(eps >= 0.f))
+    return PP_ERR_INVALID_ARG;
+  for (int o = 0; o < Co; ++o)
+    if (!(double(var[o]) + eps > 0.0)) return PP_ERR_INVALID_ARG;
+  for (int o = 0; o < Co; ++o) {
+    // y = gamma (z - mean) / sqrt(var + eps) + beta with z = conv + bias: one scale per filter, so a
+    // zero weight stays zero and the layer keeps its patterns and connectivity
+    const double scale = double(gamma[o]) / std::sqrt(double(var[o]) + double(eps));
+    float* k = w + size_t(o) * Ci * 9;
+    for (size_t t = 0; t < size_t(Ci) * 9; ++t) k[t] = float(double(k[t]) * scale);
+    bias[o] = float((double(bias[o]) - double(mean[o])) * scale + double(beta[o]));
+  }
+  return PP_OK;
+}
 
 extern "C" const char* pp_status_string(pp_status s) {
   switch (s) {

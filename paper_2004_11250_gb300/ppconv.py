@@ -56,6 +56,7 @@ _SIGS = {
     "pp_packed_info": ([_P, _P, _P, _P, _P], _I),
     "pp_packed_arrays": ([_P, _PP, _PP, _PP, _PP, _PP, _PP], _I),
     "pp_unpack_layer": ([_P, _P, _P], _I),
+    "pp_fold_batchnorm": ([_P, _P, _P, _P, _P, _P, ctypes.c_float, _I, _I], _I),
     "pp_packed_destroy": ([_P], None),
     "pp_layer_create": ([_P, _P, _P, _PP], _I),
     "pp_layer_info": ([_P, _P, _P, _P], _I),
@@ -92,6 +93,22 @@ class PPError(RuntimeError):
     def __init__(self, code: int, where: str = ""):
         super().__init__(f"{where}: {pp_status_string(code)} ({code})")
         self.code = code
+
+
+def pp_fold_batchnorm(w, bias, gamma, beta, mean, var, eps=1e-5):
+    """Batch normalisation after the conv folded into (w [Co][Ci][3][3] or [Co][Ci][9], bias [Co] or None):
+    returns new fp32 arrays (w in the shape given, bias [Co])."""
+    import numpy as np
+    w2 = np.array(w, dtype=np.float32, order="C", copy=True)
+    Co, Ci = w2.shape[0], w2.shape[1]
+    b2 = np.zeros(Co, np.float32) if bias is None else np.array(bias, dtype=np.float32, copy=True)
+    arrs = [np.ascontiguousarray(a, dtype=np.float32) for a in (gamma, beta, mean, var)]
+    for a in arrs:
+        if a.shape != (Co,):
+            raise ValueError("batch-norm parameters must have shape [Co]")
+    _check(lib.pp_fold_batchnorm(w2.ctypes.data, b2.ctypes.data, *[a.ctypes.data for a in arrs], float(eps), Co, Ci),
+           "pp_fold_batchnorm")
+    return w2, b2
 
 
 def pp_status_string(code: int) -> str:

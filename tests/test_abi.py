@@ -145,3 +145,32 @@ def test_net_shape_validation_host_only(pp):
     with pytest.raises(pp.PPError):
         pp.pp_net_finalize(net)  # no ops
     pp.pp_net_destroy(net)
+
+
+def test_fold_batchnorm_against_definition(pp, oracle_mod):
+    """pp_fold_batchnorm: conv with the folded weights and bias equals, in fp64, batch normalisation
+    (gamma (z - mean) / sqrt(var + eps) + beta per output channel) applied to the original conv z,
+    within the fp32 rounding of the folded values; zeros stay zero so the pruned layer packs the same."""
+    rng = np.random.default_rng(23)
+    Co, Ci = 12, 7
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.6, ring=False)
+    gamma = rng.uniform(-2, 2, Co).astype(np.float32)
+    beta = rng.standard_normal(Co).astype(np.float32)
+    mean = rng.standard_normal(Co).astype(np.float32)
+    var = rng.uniform(0.05, 3, Co).astype(np.float32)
+    eps = 1e-3
+    w2, b2 = pp.pp_fold_batchnorm(L.w, L.bias, gamma, beta, mean, var, eps)
+    assert ((w2.reshape(Co, Ci, 9) != 0) == (L.w.reshape(Co, Ci, 9) != 0)).all()
+    pat = oracle_mod.pattern_ids(L.w, L.mask, L.taps)
+    assert (oracle_mod.pattern_ids(w2, L.mask, L.taps) == pat).all()
+    x = rng.uniform(-1, 1, (2, Ci, 9, 11)).astype(np.float32)
+    z, _ = oracle_mod.conv_pruned(x, L.w, pat, L.taps, L.bias)
+    g = gamma.astype(np.float64) / np.sqrt(var.astype(np.float64) + eps)
+    want = (z - mean[None, :, None, None]) * g[None, :, None, None] + beta[None, :, None, None]
+    got, s2 = oracle_mod.conv_pruned(x, w2, pat, L.taps, b2)
+    # each folded weight and the bias carry one fp32 rounding (2^-24 relative)
+    assert (np.abs(got - want) <= 2.0 ** -23 * s2 + 1e-12).all()
+    # a wrong per-filter index or sign would be far outside that
+    assert np.abs(got - want).max() < 1e-5
+    with pytest.raises(pp.PPError):
+        pp.pp_fold_batchnorm(L.w, L.bias, gamma, beta, mean, -np.ones(Co, np.float32), 0.0)

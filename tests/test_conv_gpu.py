@@ -421,6 +421,21 @@ def test_direct_kernel_integer_bit_exact_and_selection(pp, runner, oracle_mod):
         wide.close()
 
 
+@pytest.mark.parametrize("kernel", ["AUTO", "REGISTER", "TMEM", "TC", "TC_FLAT", "DIRECT"])
+def test_single_pattern_layer(pp, runner, oracle_mod, kernel):
+    """Column pruning (one pattern for every kept kernel of the layer, Section 2's demo variant) is the
+    one-pattern case of the same format: every kernel that can run it matches the oracle."""
+    rng = np.random.default_rng(17)
+    taps = synth.ring8_patterns()[3:4]  # a single ring pattern, so the TMEM kernel applies too
+    Co, Ci = (130, 16) if kernel != "DIRECT" else (16, 12)
+    L = synth.make_pruned_layer(rng, Co, Ci, taps, 0.6, 0.1, 0.01)
+    assert L.taps.shape[0] == 1
+    x = rng.uniform(-1, 1, (1, Ci, 18, 22)).astype(np.float32)
+    g = run_layer(pp, runner, L, x, None, True, True, kernel=getattr(pp, "PP_KERNEL_" + kernel))
+    y, s = oracle_layer_full(oracle_mod, L, x, None, True, True)
+    check_within(g, y, s, f"single-pattern layer, {kernel}")
+
+
 def test_all_pruned_layer_gives_bias(pp, runner, oracle_mod):
     rng = np.random.default_rng(8)
     L = synth.small_random_layer(rng, 20, 10, P=8, keep=0.0)
