@@ -51,7 +51,7 @@ __device__ __forceinline__ void cp_async16(float* dst, const float* src, bool va
 }
 
 template <int CC, int FBD>
-__global__ void __launch_bounds__(DTHREADS, 2) ppconv_direct_kernel(const DirectParams p) {
+__global__ void __launch_bounds__(DTHREADS, FBD >= 16 ? 2 : 3) ppconv_direct_kernel(const DirectParams p) {
   // two stages of [CC][DTW][DPITCH] input and [CC][FBD][12] weights (9 taps padded to 12)
   extern __shared__ __align__(16) float dsm[];
   auto xs = reinterpret_cast<float(*)[CC][DTW][DPITCH]>(dsm);
