@@ -17,23 +17,28 @@
 // The dropped lo*lo term and the tf32 truncation of lo are below 2^-20 of
 // |w * x|.
 //
-// Per CTA (4 warps, one CTA per SM): M = 128 consecutive reordered filters, R
-// output rows x TW columns of pixels (R * TW = 256 TMEM columns, one fp32
-// accumulator per filter x pixel).  The K loop runs over 8-channel chunks:
-//   * weights for the chunk, 9 taps x {hi, lo} x (128 x 8) in the canonical
+// Per CTA (17 warps, one CTA per SM, persistent over tiles): warps 0-7 stage
+// the operands, warp 8 owns the TMEM (two accumulator buffers of 256 columns,
+// so one tile's epilogue overlaps the next tile's MMAs) and one of its threads
+// issues the MMAs, warps 9-16 are the epilogue.  The K loop runs over
+// 8-channel chunks, double buffered:
+//   * weights for the chunk, 9 taps x {hi, lo} x (FB x 8) in the canonical
 //     K-major layout, arrive by one bulk async copy (mbarrier transaction count);
-//   * the input tile for the chunk (R + 2 rows x TW + 2 columns, zero halo) is
-//     staged channel-innermost with cp.async, then split into hi / lo halves in
-//     place by the CTA's threads;
-//   * one thread issues 9 taps x 3 passes x R row MMAs of 128 x TW x 8.  A tap
-//     (dy, dx) is the same input tile with the operand start moved by dy rows
-//     and dx pixels (16 bytes per pixel), so no im2col copy exists;
+//   * the input box for the chunk (tile rows + 2, columns + halo, 8 channels;
+//     zero fill outside the image is the padding) arrives by a tensor-map copy
+//     (per-thread loads when x is not 16-byte aligned or W % 4 != 0), and the
+//     loader threads transpose it channel-innermost while splitting hi / lo;
+//   * a tap (dy, dx) is the same staged tile with the operand start moved by dy
+//     rows and dx pixels (16 bytes per pixel), so no im2col copy exists.
+//     Filter-major tiles (ORI_FP) run 3 MMAs per tap and row segment
+//     (w_hi x_hi, w_lo x_hi, w_hi x_lo); pixel-major tiles (ORI_PF, ORI_PFR) run
+//     2 (x_hi [w_hi | w_lo] as one 2 FB-wide operand, then x_lo w_hi);
 //   * tcgen05.commit signals an mbarrier when the chunk's MMAs have read their
 //     operands, which frees that stage for the chunk after next.
-// Epilogue: each thread owns one filter (TMEM lane); it reads its pixels with
-// tcgen05.ld and applies bias, +skip, ReLU, 2x2 max pool, storing contiguous
-// row segments.  Small grids split the chunks over a cluster and reduce the
-// accumulators through distributed shared memory in rank order.
+// Epilogue: bias, +skip, ReLU, 2x2 max pool from tcgen05.ld, stores to each
+// filter's original channel.  This kernel has no channel split: layers with
+// more than 64 filters on maps at most 128 wide can also run the flat kernel
+// (conv_tcf.cu), which splits the chunks of small grids over a cluster.
 //
 // Every wait on an mbarrier is bounded; on timeout the kernel records an error
 // in the layer's device status word and skips the rest of its work.

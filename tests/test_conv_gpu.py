@@ -119,7 +119,7 @@ def test_tensor_core_kernel(pp, runner, oracle_mod, case, flags):
 
 
 def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
-    """Shapes that exercise every tile width (16/32/64/128 pixels) and the cluster split of the channel chunks."""
+    """Shapes that exercise every tile width (16/32/64/128 pixels), ragged blocks and persistent CTAs with several tiles."""
     rng = np.random.default_rng(31)
     for (N, Ci, Co, H, W) in ((1, 72, 130, 12, 14), (1, 40, 64, 20, 30), (1, 24, 128, 9, 60), (1, 16, 33, 5, 140),
                               (2, 136, 200, 7, 9)):
