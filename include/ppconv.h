@@ -196,7 +196,8 @@ pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* 
  *                       16 filters per thread; layers with at most 16 input
  *                       or at most 16 output channels (first and last layers).
  * PP_KERNEL_AUTO picks by an estimate of each kernel's time for the layer's
- * density.  Setting a kernel the layer cannot run returns PP_ERR_UNSUPPORTED. */
+ * density (the direct kernel for Ci <= 4).  Setting a kernel the layer cannot
+ * run returns PP_ERR_UNSUPPORTED. */
 #define PP_KERNEL_AUTO 0
 #define PP_KERNEL_TMEM 1
 #define PP_KERNEL_REGISTER 2
@@ -206,9 +207,10 @@ pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* 
 pp_status pp_layer_set_kernel(pp_layer* layer, int kernel);
 /* The kernel that pp_conv_forward will run (one of the PP_KERNEL_ values above, not _AUTO). */
 pp_status pp_layer_kernel(const pp_layer* layer, int* kernel);
-/* Time every kernel that can run this layer on zero-filled scratch tensors of
- * the given shape and flags (a few launches each, on stream, synchronous) and
- * keep the fastest for the layer; the flat tensor-core kernel is timed at the
+/* Time the kernels that can run this layer (tensor-core, TMEM and direct
+ * kernels where their layouts exist; the register kernel only when none of
+ * them can) on zero-filled scratch tensors of the given shape and flags (a few
+ * launches each, on stream, synchronous) and keep the fastest for the layer; the flat tensor-core kernel is timed at the
  * best few tile geometries (rows per tile, cluster split) of its cost model and
  * keeps the winning one for launches of this shape.  The kernels differ in speed by layer shape:
  * the tensor-core kernel needs many output tiles to fill the GPU, the FMA

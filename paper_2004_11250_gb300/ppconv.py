@@ -231,7 +231,7 @@ def pp_conv_forward(layer, x, y, skip, N, H, W, flags, stream=None):
 
 
 def pp_conv_forward_noalloc(layer, x, y, skip, N, H, W, flags, stream=None):
-    """pp_conv_forward through the flat tensor-core kernel with a static split workspace (no device allocation)."""
+    """pp_conv_forward through the flat tensor-core kernel, whose split reduction needs no workspace (no device allocation)."""
     _check(lib.pp_conv_forward_noalloc(layer, _dp(x), _dp(y), _dp(skip), N, H, W, flags, _stream(stream)),
            "pp_conv_forward_noalloc")
 
