@@ -532,6 +532,27 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               }
             }
             tm_wait_ld();
+            // residual (no pool): the 16 skip values are added in a pass of their
+            // own, with no store between the loads, so their latencies overlap.
+            // The condition is warp-uniform (kernel arguments): every lane takes
+            // part in the shuffles.  Every lane loads (lanes without an output
+            // from the tensor's first element) and masks the value, so the 16
+            // loads are unconditional and independent.
+            if (sbase && !pool) {
+#pragma unroll
+              for (int k0 = 0; k0 < 16; k0 += 8) {
+                float sv[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                  const int o = __shfl_sync(0xffffffffu, pm[(jj + k0 + k) >> 5], (jj + k0 + k) & 31);
+                  const bool use = o >= 0 && in0;
+                  sv[k] = __ldg(sbase + (use ? o * HW + roff : 0));
+                  sv[k] = use ? sv[k] : 0.f;
+                }
+#pragma unroll
+                for (int k = 0; k < 8; ++k) a[k0 + k] += sv[k];
+              }
+            }
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
               const int j = jj + k;
@@ -539,7 +560,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               const float bs = __shfl_sync(0xffffffffu, bv[j >> 5], j & 31);
               if (o < 0) continue;  // past the last filter: the same for every lane
               float v = a[k] + bs;
-              if (sbase && in0) v += __ldg(sbase + o * HW + roff);
+              if (sbase && pool && in0) v += __ldg(sbase + o * HW + roff);
               if (p.flags & PP_RELU) v = fmaxf(v, 0.f);
               if (!pool) {
                 if (in0) ybase[o * HW + roff] = v;
