@@ -469,13 +469,23 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         // this CTA's partial tile into its own shared memory (free once the
         // accumulators are ready): row m of [128][ncols + 4], padded so a warp's
         // 16-byte stores to 32 rows spread over the banks
+        // (4 TMEM loads per wait; the bounds are warp-uniform, as the
+        // warp-collective loads require)
         float* prow = reinterpret_cast<float*>(smem) + m * (p.ncols + 4);
-        for (int cb = half * 8; cb < p.ncols; cb += 16) {
-          float a[8];
-          tm_ld8(lanebase + (uint32_t)cb, a);
+        for (int cb0 = half * 8; cb0 < p.ncols; cb0 += 64) {
+          float a[4][8];
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            if (cb0 + 16 * u < p.ncols) tm_ld8(lanebase + (uint32_t)(cb0 + 16 * u), a[u]);
           tm_wait_ld();
-          *reinterpret_cast<float4*>(prow + cb) = make_float4(a[0], a[1], a[2], a[3]);
-          *reinterpret_cast<float4*>(prow + cb + 4) = make_float4(a[4], a[5], a[6], a[7]);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int cb = cb0 + 16 * u;
+            if (cb < p.ncols) {
+              *reinterpret_cast<float4*>(prow + cb) = make_float4(a[u][0], a[u][1], a[u][2], a[u][3]);
+              *reinterpret_cast<float4*>(prow + cb + 4) = make_float4(a[u][4], a[u][5], a[u][6], a[u][7]);
+            }
+          }
         }
       } else {
         const int jr = T.fb * FB + m;
