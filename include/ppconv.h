@@ -242,6 +242,24 @@ pp_status pp_layer_pin_flat_geometry(pp_layer* layer, int N, int H, int W, int f
  * bounded wait (its output is then invalid); the word is cleared by the read. */
 pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);
 
+/* Polls of an mbarrier after which a wait in the tensor-core kernels gives up:
+ * the kernel then sets the layer's device status word, skips the rest of its
+ * work, waits (with the same bound) for its own copies in flight and exits.
+ * A poll that finds the phase incomplete suspends the thread for a few
+ * microseconds (3.8 us measured on GB300 with pp_wait_probe), so a wait gives
+ * up after about a second; the longest wait of a correct launch is below a
+ * millisecond. */
+#define PP_WAIT_POLLS (1L << 18)
+
+/* Diagnostic for the bound above.  One thread polls an mbarrier that nothing
+ * completes, with the kernels' poll instruction, `polls` times (1 .. 2^20),
+ * and reports *gave_up = 1 and the elapsed device time in ns; a full wait
+ * takes about PP_WAIT_POLLS / polls times as long.  Synchronous, on the legacy
+ * default stream; allocates 16 bytes of device memory for the results.
+ * Errors: PP_ERR_INVALID_ARG (null pointer, polls out of range), PP_ERR_OOM,
+ * PP_ERR_CUDA. */
+pp_status pp_wait_probe(long long polls, int* gave_up, long long* elapsed_ns);
+
 void pp_layer_destroy(pp_layer* layer);
 
 /* ------------------------------------------------------------------------

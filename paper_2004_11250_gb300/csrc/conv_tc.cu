@@ -67,7 +67,7 @@ constexpr int EPI_WARP0 = 9;       // warps 9-16: epilogue, two per TMEM lane qu
 constexpr int NEPI = 256;          // epilogue threads
 constexpr int NTHREADS = 544;
 constexpr int LBATCH = 4;          // loader items whose global loads are in flight together
-constexpr long WAIT_LIMIT = 1L << 22;  // mbarrier polls before a wait gives up
+constexpr long WAIT_LIMIT = PP_WAIT_POLLS;  // mbarrier polls before a wait gives up
 
 // Orientation of the GEMM on the tensor core.
 //   ORI_FP: M = 128 filters, N = TW pixels of one output row (narrow maps)
@@ -823,3 +823,47 @@ pp_status tc_status(const TcLayout& T, int* device_error) {
 }
 
 }  // namespace ppc
+
+namespace {
+
+// One thread polls an mbarrier that nothing ever completes, with the poll of
+// the kernels' bounded waits, `polls` times, and records that it gave up and
+// how long the polls took (globaltimer, ns).
+__global__ void wait_probe_kernel(long long polls, int* gave_up, long long* ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(su32(&bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint64_t t0, t1;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0)::"memory");
+    bool done = false;
+    for (long long i = 0; i < polls && !done; ++i) done = mbar_try(su32(&bar), 0u);
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t1)::"memory");
+    *gave_up = done ? 0 : 1;
+    *ns = (long long)(t1 - t0);
+  }
+}
+
+}  // namespace
+
+extern "C" pp_status pp_wait_probe(long long polls, int* gave_up, long long* elapsed_ns) {
+  if (!gave_up || !elapsed_ns || polls < 1 || polls > (1LL << 20)) return PP_ERR_INVALID_ARG;
+  void* d = nullptr;
+  if (cudaMalloc(&d, 16) != cudaSuccess) {
+    cudaGetLastError();
+    return PP_ERR_OOM;
+  }
+  long long* d_ns = static_cast<long long*>(d);
+  int* d_gave = reinterpret_cast<int*>(static_cast<unsigned char*>(d) + 8);
+  wait_probe_kernel<<<1, 32>>>(polls, d_gave, d_ns);
+  long long h[2] = {0, 0};
+  const bool ok = cudaGetLastError() == cudaSuccess && cudaMemcpy(h, d, 16, cudaMemcpyDeviceToHost) == cudaSuccess;
+  cudaFree(d);
+  if (!ok) return PP_ERR_CUDA;
+  *elapsed_ns = h[0];
+  *gave_up = (int)(h[1] & 0xFFFFFFFF);
+  return PP_OK;
+}

@@ -65,7 +65,7 @@ constexpr int IN_MAX = 2 * PIX_MAX * 16;  // largest hi (or lo) operand of one c
 constexpr int SMEM_ALLOC = 231424;    // dynamic shared memory (static use stays below 1 KB)
 constexpr int SMEM_USE = SMEM_ALLOC - 1024;  // after aligning the base to 1024
 constexpr int ITEMS_MAX = (2 * PIX_MAX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
-constexpr long WAIT_LIMIT = 1L << 22;
+constexpr long WAIT_LIMIT = PP_WAIT_POLLS;  // mbarrier polls before a wait gives up
 constexpr int MAX_SPLIT = 16;
 static_assert(2 * (W_BYTES + 2 * IN_MAX) <= SMEM_USE, "shared memory plan");
 static_assert(FB * NMAX * 4 <= SMEM_USE, "split reduction buffer");

@@ -40,6 +40,8 @@ PP_KERNEL_TC = 3
 PP_KERNEL_TC_FLAT = 4
 PP_KERNEL_DIRECT = 5
 
+PP_WAIT_POLLS = 1 << 18
+
 PP_ADD_SKIP = 1
 PP_RELU = 2
 PP_POOL2 = 4
@@ -65,6 +67,7 @@ _SIGS = {
     "pp_layer_set_kernel": ([_P, _I], _I),
     "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_device_status": ([_P, _P], _I),
+    "pp_wait_probe": ([ctypes.c_longlong, _P, _P], _I),
     "pp_layer_autotune": ([_P, _I, _I, _I, _I, _P], _I),
     "pp_layer_flat_geometry": ([_P, _I, _I, _I, _I, _P, _P], _I),
     "pp_layer_pin_flat_geometry": ([_P, _I, _I, _I, _I, _I, _I], _I),
@@ -265,6 +268,13 @@ def pp_layer_device_status(layer) -> int:
     v = _I()
     _check(lib.pp_layer_device_status(layer, ctypes.byref(v)), "pp_layer_device_status")
     return v.value
+
+
+def pp_wait_probe(polls: int):
+    """(gave_up, elapsed_ns) of `polls` polls of an mbarrier that nothing completes (see the header)."""
+    g, ns = _I(), ctypes.c_longlong()
+    _check(lib.pp_wait_probe(polls, ctypes.byref(g), ctypes.byref(ns)), "pp_wait_probe")
+    return g.value, ns.value
 
 
 def pp_layer_destroy(layer):

@@ -174,3 +174,11 @@ def test_fold_batchnorm_against_definition(pp, oracle_mod):
     assert np.abs(got - want).max() < 1e-5
     with pytest.raises(pp.PPError):
         pp.pp_fold_batchnorm(L.w, L.bias, gamma, beta, mean, -np.ones(Co, np.float32), 0.0)
+
+
+def test_wait_probe_rejects_bad_arguments(pp):
+    """Argument checks come before any device work (this runs without a GPU)."""
+    for polls in (0, -1, (1 << 20) + 1):
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_wait_probe(polls)
+        assert e.value.code == pp.PP_ERR_INVALID_ARG

@@ -560,3 +560,20 @@ def test_bad_arguments_rejected(pp, runner):
         assert e.value.code == pp.PP_ERR_INVALID_ARG
     finally:
         L.close()
+
+
+def test_bounded_wait_gives_up_and_device_stays_usable(pp, runner, oracle_mod):
+    """A wait that nothing completes (the poll of the tensor-core kernels' waits, on an mbarrier nobody
+    arrives on) gives up and says so; a full wait of PP_WAIT_POLLS polls is bounded in time; the context
+    stays usable (a tensor-core conv right after is within the bound)."""
+    gave_up, ns = pp.pp_wait_probe(1024)
+    assert gave_up == 1 and ns > 0
+    full_wait_s = ns / 1024 * pp.PP_WAIT_POLLS / 1e9
+    print(f"one poll {ns / 1024:.1f} ns; a full wait gives up after ~{full_wait_s:.2f} s")
+    assert full_wait_s < 5.0
+    rng = np.random.default_rng(404)
+    L = synth.small_random_layer(rng, 40, 24, P=8, keep=0.4)
+    x = rng.uniform(-1, 1, (1, 24, 12, 20)).astype(np.float32)
+    g = run_layer(pp, runner, L, x, None, True, False, kernel=pp.PP_KERNEL_TC)
+    y, s = oracle_layer_full(oracle_mod, L, x, None, True, False)
+    check_within(g, y, s, "tensor-core conv after a given-up wait")
