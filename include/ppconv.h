@@ -311,7 +311,11 @@ pp_status pp_net_output_shape(const pp_net* net, int* N, int* C, int* H, int* W)
 /* With enable != 0, pp_net_run captures its launches into a CUDA graph on the
  * first call for a given (x, y, stream) and replays that graph afterwards (one
  * host launch per run).  Needs a non-NULL stream; with the legacy default
- * stream the ops are launched one by one.  Default: off. */
+ * stream the ops are launched one by one.  Default: off.  A graph keeps the
+ * kernels and tile geometries the layers had when it was captured; every call
+ * of this function drops the captured graphs, so calling it again after
+ * changing a borrowed layer (pp_layer_set_kernel, pins) makes the next run
+ * capture the change. */
 pp_status pp_net_use_graph(pp_net* net, int enable);
 
 /* Device-resident run: x and y are device buffers of the input and output
@@ -322,7 +326,10 @@ pp_status pp_net_run(pp_net* net, const float* x, float* y, void* stream);
  * End-to-end run on host buffers: copies x_host to the device, runs the
  * network and copies the output to y_host, all on stream, and synchronises
  * the stream before returning.  Pinned host memory gives overlap-free DMA at
- * full speed; pageable memory works too.
+ * full speed; pageable memory works too.  With graphs enabled, a non-NULL
+ * stream and page-locked x_host and y_host, the two copies and the ops are one
+ * CUDA graph, captured on the first call for those buffers and stream and
+ * replayed afterwards (one host launch per frame).
  */
 pp_status pp_net_run_host(pp_net* net, const float* x_host, float* y_host, void* stream);
 

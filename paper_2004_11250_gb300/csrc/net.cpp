@@ -42,6 +42,11 @@ struct pp_net {
   const float* g_x = nullptr;
   float* g_y = nullptr;
   cudaStream_t g_stream = nullptr;
+  // pp_net_run_host with pinned buffers: the two copies and the ops in one graph
+  cudaGraphExec_t hexec = nullptr;
+  const float* h_x = nullptr;
+  float* h_y = nullptr;
+  cudaStream_t h_stream = nullptr;
 };
 
 
@@ -219,6 +224,11 @@ extern "C" pp_status pp_net_output_shape(const pp_net* net, int* N, int* C, int*
 extern "C" pp_status pp_net_use_graph(pp_net* net, int enable) {
   if (!net) return PP_ERR_INVALID_ARG;
   net->use_graph = enable != 0;
+  // drop the captured graphs: the next runs capture the layers' current kernels
+  if (net->gexec) cudaGraphExecDestroy(net->gexec);
+  if (net->hexec) cudaGraphExecDestroy(net->hexec);
+  net->gexec = nullptr;
+  net->hexec = nullptr;
   return PP_OK;
 }
 
@@ -253,6 +263,20 @@ extern "C" pp_status pp_net_run(pp_net* net, const float* x, float* y, void* str
   return cudaGraphLaunch(net->gexec, stream) == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
+namespace {
+
+// True for page-locked host memory (cudaHostAlloc / cudaHostRegister).
+bool is_pinned(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeHost;
+}
+
+}  // namespace
+
 extern "C" pp_status pp_net_run_host(pp_net* net, const float* x_host, float* y_host, void* stream_) {
   if (!net || !x_host || !y_host || !net->finalized) return PP_ERR_INVALID_ARG;
   cudaStream_t stream = (cudaStream_t)stream_;
@@ -266,6 +290,43 @@ extern "C" pp_status pp_net_run_host(pp_net* net, const float* x_host, float* y_
       return PP_ERR_OOM;
     }
   }
+  // With graphs on and page-locked host buffers, the input copy, the ops and
+  // the output copy are captured once per (x_host, y_host, stream) and each
+  // call is one graph launch; otherwise they are issued one by one.
+  if (net->use_graph && stream != nullptr && is_pinned(x_host) && is_pinned(y_host)) {
+    if (!net->hexec || net->h_x != x_host || net->h_y != y_host || net->h_stream != stream) {
+      if (net->hexec) {
+        cudaGraphExecDestroy(net->hexec);
+        net->hexec = nullptr;
+      }
+      cudaGraph_t g = nullptr;
+      if (cudaStreamBeginCapture(stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) return PP_ERR_CUDA;
+      pp_status st = PP_OK;
+      if (cudaMemcpyAsync(net->d_in, x_host, in_bytes, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        st = PP_ERR_CUDA;
+      if (st == PP_OK) st = run_ops(net, net->d_in, net->d_out, stream);
+      if (st == PP_OK &&
+          cudaMemcpyAsync(y_host, net->d_out, out_bytes, cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+        st = PP_ERR_CUDA;
+      cudaError_t ce = cudaStreamEndCapture(stream, &g);
+      if (st != PP_OK || ce != cudaSuccess) {
+        if (g) cudaGraphDestroy(g);
+        cudaGetLastError();
+        return st != PP_OK ? st : PP_ERR_CUDA;
+      }
+      ce = cudaGraphInstantiate(&net->hexec, g, 0);
+      cudaGraphDestroy(g);
+      if (ce != cudaSuccess) {
+        net->hexec = nullptr;
+        return PP_ERR_CUDA;
+      }
+      net->h_x = x_host;
+      net->h_y = y_host;
+      net->h_stream = stream;
+    }
+    if (cudaGraphLaunch(net->hexec, stream) != cudaSuccess) return PP_ERR_CUDA;
+    return cudaStreamSynchronize(stream) == cudaSuccess ? PP_OK : PP_ERR_CUDA;
+  }
   if (cudaMemcpyAsync(net->d_in, x_host, in_bytes, cudaMemcpyHostToDevice, stream) != cudaSuccess)
     return PP_ERR_CUDA;
   pp_status st = pp_net_run(net, net->d_in, net->d_out, stream_);
@@ -278,6 +339,7 @@ extern "C" pp_status pp_net_run_host(pp_net* net, const float* x_host, float* y_
 extern "C" void pp_net_destroy(pp_net* net) {
   if (!net) return;
   if (net->gexec) cudaGraphExecDestroy(net->gexec);
+  if (net->hexec) cudaGraphExecDestroy(net->hexec);
   for (float* p : net->buffers) cudaFree(p);
   cudaFree(net->d_in);
   cudaFree(net->d_out);

@@ -577,3 +577,42 @@ def test_bounded_wait_gives_up_and_device_stays_usable(pp, runner, oracle_mod):
     g = run_layer(pp, runner, L, x, None, True, False, kernel=pp.PP_KERNEL_TC)
     y, s = oracle_layer_full(oracle_mod, L, x, None, True, False)
     check_within(g, y, s, "tensor-core conv after a given-up wait")
+
+
+def test_run_host_graph_and_plain_paths(pp, runner):
+    """pp_net_run_host on a non-default stream: page-locked buffers take the captured graph (copies and ops
+    in one graph, replayed on the second call and re-captured for other buffers), pageable buffers the
+    op-by-op path, and graphs off the plain path; all give the device run's output bit for bit."""
+    for spec in (synth.cfg0_single(), synth.cfg2_style()):
+        run_host_paths(pp, runner, spec)
+
+
+def run_host_paths(pp, runner, spec):
+    dn = runner.DeviceNet(spec, use_graph=True)
+    try:
+        s = torch.cuda.Stream()
+        x = torch.from_numpy(spec.x).cuda()
+        ref = torch.empty(dn.out_shape, device="cuda")
+        dn.run(x, ref, s)
+        s.synchronize()
+        ref = ref.cpu()
+        outs = []
+        xh = torch.from_numpy(spec.x).pin_memory()
+        for _ in range(2):
+            yh = torch.full(dn.out_shape, float("nan")).pin_memory()
+            dn.run_host(xh, yh, s)
+            outs.append(yh)
+        yh2 = torch.full(dn.out_shape, float("nan")).pin_memory()  # other buffers: captured again
+        dn.run_host(xh, yh2, s)
+        outs.append(yh2)
+        yp = torch.full(dn.out_shape, float("nan"))  # pageable: copies issued one by one
+        dn.run_host(torch.from_numpy(spec.x.copy()), yp, s)
+        outs.append(yp)
+        pp.pp_net_use_graph(dn.net, False)
+        yo = torch.full(dn.out_shape, float("nan")).pin_memory()
+        dn.run_host(xh, yo, s)
+        outs.append(yo)
+        for o in outs:
+            assert torch.equal(o, ref)
+    finally:
+        dn.close()
