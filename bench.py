@@ -17,10 +17,11 @@ Printed JSON line (rank 0):
              that run on the tensor cores (3xTF32 dense-tap FLOPs executed vs
              the measured bf16 peak x the nominal tf32 / bf16 ratio)
   cpu_baseline the fp64 CPU oracle on this host's cores on a bounded sample
-  configs    ms/frame, GFLOP/s and roofline fraction of all five workloads
+  configs    ms/frame, GFLOP/s, roofline fraction and tensor-pipe view of all
+             five workloads
 
-``--impl reference`` times the CPU oracle alone (the reference arm of this
-build: the paper ships no code) and prints the same metric.
+``--impl reference`` times the CPU oracle alone (the reference arm: the paper
+ships no code) and prints the same metric.
 """
 from __future__ import annotations
 
@@ -278,6 +279,22 @@ def kernel_source_hash():
     return h.hexdigest()
 
 
+def tensor_view(shapes, kern, op_ms, pruned):
+    """Tensor-pipe view of the pruned ops that run on a tensor-core kernel: their dense 9-tap contraction
+    in 3 tf32 passes (hi*hi, lo*hi, hi*lo) per second against the tf32 peak; None without such ops."""
+    tc_ops = [k for k in pruned if kern[k] in ("ppconv_tc_kernel", "ppconv_tcf_kernel")]
+    if not tc_ops:
+        return None
+    tf = sum(3 * 2 * shapes[k]["N"] * shapes[k]["Ci"] * shapes[k]["Co"] * 9 * shapes[k]["H"] * shapes[k]["W"]
+             for k in tc_ops)
+    tt = sum(op_ms[k] for k in tc_ops) * 1e-3
+    bpk, bsrc = bf16_peak_tflops()
+    tpk = bpk * TF32_PER_BF16
+    return {"bound": "tensor", "ops": len(tc_ops), "achieved": round(tf / tt / 1e12, 2), "peak": round(tpk, 1),
+            "unit": "TFLOP/s (tf32, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
+            "peak_source": f"{bsrc} bf16 {bpk} TFLOP/s x nominal tf32/bf16 {TF32_PER_BF16:.3f}"}
+
+
 def bench_config(name, steps, warmup, flush, stream, hbm):
     """ms/frame, GFLOP/s and per-op roofline fractions of one workload (used for the all-configs table)."""
     import torch
@@ -297,10 +314,13 @@ def bench_config(name, steps, warmup, flush, stream, hbm):
         pr = [f for s, f in zip(shapes, fr) if s["pruned"]]
         del acts
         from paper_2004_11250_gb300 import ppconv as pp
-        kern = sorted(set(KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") for L in dn.layers if not L.dense))
+        per_op = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "dense" for L in dn.layers]
+        kern = sorted(set(k for k in per_op if k != "dense"))
+        tv = tensor_view(shapes, per_op, op_ms, [k for k, s in enumerate(shapes) if s["pruned"]])
         return {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1), "kernels": kern,
                 "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
-                "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None}
+                "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None,
+                "tensor_tflops": tv["achieved"] if tv else None, "tensor_frac": tv["frac"] if tv else None}
     finally:
         dn.close()
 
@@ -505,18 +525,7 @@ def main():
             R, S = pp.pp_layer_flat_geometry(L.handle, sh["N"], sh["H"], sh["W"], runner.op_flags(op))
             g = f"{R}:{S}" if R else "model"
         geo.append(g)
-    tc_ops = [k for k in pruned if kern[k] in ("ppconv_tc_kernel", "ppconv_tcf_kernel")]
-    tensor = None
-    if tc_ops:
-        # 3 tf32 products per dense tap MAC: hi*hi, lo*hi, hi*lo
-        tf = sum(3 * 2 * shapes[k]["N"] * shapes[k]["Ci"] * shapes[k]["Co"] * 9 * shapes[k]["H"] * shapes[k]["W"]
-                 for k in tc_ops)
-        tt = sum(op_ms[k] for k in tc_ops) * 1e-3
-        bpk, bsrc = bf16_peak_tflops()
-        tpk = bpk * TF32_PER_BF16
-        tensor = {"bound": "tensor", "ops": len(tc_ops), "achieved": round(tf / tt / 1e12, 2), "peak": round(tpk, 1),
-                  "unit": "TFLOP/s (tf32, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
-                  "peak_source": f"{bsrc} bf16 {bpk} TFLOP/s x nominal tf32/bf16 {TF32_PER_BF16:.3f}"}
+    tensor = tensor_view(shapes, kern, op_ms, pruned)
     # the dominant kernel (most device time over the pruned ops): its surviving FLOPs per launch over
     # its mean launch duration, against the FP32 roofline of the method
     by_kern = {}
