@@ -44,6 +44,7 @@ if ROOT not in sys.path:
 HBM_PEAK_GBS_FALLBACK = 6800.0
 BF16_PEAK_TFLOPS_FALLBACK = 1900.0
 TF32_PER_BF16 = 1.1 / 2.25  # nominal dense tensor rates
+CONFIG_CPU_SECONDS = 4.0  # oracle sample per workload of the all-configs table
 KERNEL_NAMES = {1: "ppconv_tm_kernel", 2: "ppconv_kernel", 3: "ppconv_tc_kernel", 4: "ppconv_tcf_kernel",
                 5: "ppconv_direct_kernel"}
 SM_COUNT = 152
@@ -158,20 +159,30 @@ class ClockSampler:
 
 def cpu_oracle_sample(spec, target_s: float, seed: int = 0):
     """Time the fp64 oracle on a bounded sample of the workload: every op, restricted to its first
-    ceil(f * Co) filters, on a seeded input of the op's input shape.  f is calibrated on the first
+    ceil(f * Co) filters (at least one per oracle thread), on a seeded input of the op's input shape
+    (one per distinct shape).  f is calibrated on the first
     pruned op so that the whole sample takes about target_s seconds.  Returns (GFLOP/s, f, seconds)."""
     from oracle import oracle as orc
     from paper_2004_11250_gb300 import synth
     rng = np.random.default_rng(seed)
     shapes = op_shapes(spec)
     total_flops = sum(s["flops"] for s in shapes)
-    inputs = [rng.uniform(-1, 1, (s["N"], s["Ci"], s["H"], s["W"])).astype(np.float32) for s in shapes]
+    by_shape = {}  # one seeded input per distinct input shape (the timing does not depend on the values)
+    inputs = []
+    for s in shapes:
+        key = (s["N"], s["Ci"], s["H"], s["W"])
+        if key not in by_shape:
+            by_shape[key] = rng.uniform(-1, 1, key).astype(np.float32)
+        inputs.append(by_shape[key])
     pats = [orc.pattern_ids(op.layer.w, op.layer.mask, op.layer.taps) if isinstance(op.layer, synth.PrunedLayer)
             else None for op in spec.ops]
 
+    nthr = max(1, orc.num_threads())
+
     def run(k, f):
+        # at least one filter per oracle thread (it runs in parallel over images and filters)
         L = spec.ops[k].layer
-        co = max(1, int(math.ceil(f * L.Co)))
+        co = min(L.Co, max(nthr, int(math.ceil(f * L.Co))))
         t0 = time.perf_counter()
         if pats[k] is not None:
             orc.conv_pruned(inputs[k], L.w[:co], pats[k][:co], L.taps, None if L.bias is None else L.bias[:co])
@@ -182,7 +193,7 @@ def cpu_oracle_sample(spec, target_s: float, seed: int = 0):
         return dt, s["flops"] * co / s["Co"]
 
     k0 = max(range(len(shapes)), key=lambda k: shapes[k]["flops"])
-    f0 = min(1.0, 2.0 / max(1, shapes[k0]["Co"]))
+    f0 = min(1.0, nthr / max(1, shapes[k0]["Co"]))
     dt, fl = run(k0, f0)
     rate = fl / max(dt, 1e-9)
     f = min(1.0, target_s * rate / total_flops)
@@ -564,8 +575,22 @@ def main():
         from oracle import oracle as orc
         v, f, secs = cpu_oracle_sample(spec, args.cpu_seconds)
         cpu = {"value": round(v, 3), "unit": "GFLOP/s", "cores": orc.num_threads(), "kind": "oracle",
-               "sample": (f"every op on its first {f:.4f} of filters (seeded inputs), {secs:.1f} s" if f < 1 else
+               "sample": (f"every op on its first {f:.4f} of filters, at least one per thread (seeded inputs), {secs:.1f} s" if f < 1 else
                           f"{f:.0f} whole frames of every op (seeded inputs), {secs:.1f} s")}
+        if configs is not None:
+            # the oracle beside every workload, same cores, a bounded sample each (the sweep: its middle point)
+            from paper_2004_11250_gb300 import synth
+            for name in configs:
+                if name == args.workload:
+                    cv, cf, cs = v, f, secs
+                else:
+                    cspec = synth.cfg4_point(256, 8, 0.35) if name == "sweep" else workload(name)
+                    cv, cf, cs = cpu_oracle_sample(cspec, CONFIG_CPU_SECONDS)
+                configs[name]["cpu_oracle"] = {
+                    "gflops": round(cv, 3), "cores": orc.num_threads(),
+                    "sample": ("sweep point C256 P8 keep 0.35: " if name == "sweep" else "")
+                    + (f"every op on its first {cf:.4f} of filters (at least one per thread), {cs:.1f} s" if cf < 1 else
+                       f"{cf:.0f} whole frames, {cs:.1f} s")}
 
     if rank == 0:
         line = {
