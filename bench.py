@@ -426,7 +426,8 @@ def run_reference(args, ws, rank):
         "config": config_dict(args.workload),
         "cpu_baseline": {"value": round(value, 3), "unit": "GFLOP/s", "cores": orc.num_threads(), "kind": "oracle",
                          "sample": f"per step: every op of the workload on {statistics.median(fs):.4f} of its filters "
-                                   f"(frames when >= 1), seeded inputs; {wall:.1f} s for {args.steps} steps"},
+                                   f"(at least one per oracle thread; frames when >= 1), seeded inputs; "
+                                   f"{wall:.1f} s for {args.steps} steps"},
         "e2e": {"value": round(value, 3), "unit": "GFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
