@@ -30,7 +30,10 @@
  *     unless stated.  Launch errors are returned by the call; faults that
  *     happen later surface at the caller's next synchronisation.
  *   - Activation, skip and output pointers are caller-owned device memory,
- *     dense NCHW fp32, 16-byte aligned.  An output must not overlap an input.
+ *     dense NCHW fp32.  Outputs must be 16-byte aligned and inputs at least
+ *     4-byte aligned (a 16-byte aligned input with W a multiple of 4 takes the
+ *     faster bulk-copy paths); others are rejected with PP_ERR_INVALID_ARG.
+ *     An output must not overlap an input.
  *   - A handle may be used from one host thread at a time.
  */
 #ifndef PPCONV_H
@@ -150,9 +153,9 @@ pp_status pp_layer_info(const pp_layer* layer, int* Co, int* Ci, int64_t* device
  *   x     [N][Ci][H][W] device input
  *   y     [N][Co][H][W], or [N][Co][H/2][W/2] with PP_POOL2 (H, W even)
  *   skip  [N][Co][H][W] device tensor added before the ReLU (PP_ADD_SKIP), else NULL
- * Errors: PP_ERR_INVALID_ARG (null pointer, N/H/W < 1, flags), PP_ERR_UNSUPPORTED
- *   (PP_POOL2 with odd H or W, or a pattern the kernels do not cover),
- *   PP_ERR_CUDA (launch failure).
+ * Errors: PP_ERR_INVALID_ARG (null pointer, N/H/W < 1, flags, y not 16-byte
+ *   or x not 4-byte aligned), PP_ERR_UNSUPPORTED (PP_POOL2 with odd H or W, or
+ *   a pattern the kernels do not cover), PP_ERR_CUDA (launch failure).
  */
 pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H, int W,
                           int flags, void* stream);
