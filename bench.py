@@ -11,11 +11,14 @@ Printed JSON line (rank 0):
   ms_per_step  ms per frame
   e2e        the same metric through pp_net_run_host (pinned host buffers,
              H2D + run + D2H + sync every step)
-  roofline   the pruned convs: surviving-weight TFLOP/s over their launches vs
-             the FP32 FMA peak 152 SM x 128 lanes x 2 FLOP x 2.07 GHz (the
-             method's roofline); "tensor" adds the tensor-pipe view of the ops
-             that run on the tensor cores (3xTF32 dense-tap FLOPs executed vs
-             the measured bf16 peak x the nominal tf32 / bf16 ratio)
+  roofline   the dominant kernel of the pruned convs: its surviving-weight
+             TFLOP/s over its launches timed inside the frame (op by op, events
+             between the ops, L2 flushed once per frame) vs the FP32 FMA peak
+             measured by pp_peak_probe in the same run (the method's roofline;
+             the derived SMs x 128 lanes x 2 FLOP x max clock beside it);
+             "tensor" adds the tensor-pipe view of the ops that run on the
+             tensor cores (dense-tap FLOPs executed in their passes vs the
+             tcgen05 MMA peak measured by the same probe)
   cpu_baseline the fp64 CPU oracle on this host's cores on a bounded sample
   configs    ms/frame, GFLOP/s, roofline fraction and tensor-pipe view of all
              five workloads
@@ -42,16 +45,38 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 HBM_PEAK_GBS_FALLBACK = 6800.0
-BF16_PEAK_TFLOPS_FALLBACK = 1900.0
-TF32_PER_BF16 = 1.1 / 2.25  # nominal dense tensor rates
 CONFIG_CPU_SECONDS = 4.0  # oracle sample per workload of the all-configs table
 KERNEL_NAMES = {1: "ppconv_tm_kernel", 2: "ppconv_kernel", 3: "ppconv_tc_kernel", 4: "ppconv_tcf_kernel",
                 5: "ppconv_direct_kernel"}
-SM_COUNT = 152
 FP32_LANES_PER_SM = 128
 SM_MAX_MHZ = 2070.0
-FP32_PEAK_TFLOPS = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12  # 80.55
 L2_FLUSH_BYTES = 512 << 20
+# Roofline denominators: FP32 FMA peak in TFLOP/s.  bench.py replaces it by the rate pp_peak_probe
+# measures on the GPU it runs on (set_fp32_peak); the value below is the derived peak of a 152-SM
+# GB300 at its maximum clock (152 x 128 lanes x 2 FLOP x 2.07 GHz), used before that and on the CPU.
+FP32_PEAK_TFLOPS = 152 * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12  # 80.55
+
+
+def set_fp32_peak(tflops: float):
+    global FP32_PEAK_TFLOPS
+    FP32_PEAK_TFLOPS = float(tflops)
+
+
+def measure_peaks():
+    """FP32 FMA and tcgen05 MMA (tf32, f16) peaks of this GPU by pp_peak_probe, each the best of 3
+    launches of a few milliseconds, with the SM clock seen during the best one; plus the derived FP32
+    peak (SMs x 128 lanes x 2 FLOP x maximum clock)."""
+    import torch
+    from paper_2004_11250_gb300 import ppconv as pp
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    out = {"sms": sms, "derived_fp32_tflops": round(sms * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12, 2),
+           "derived_from": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x 2 FLOP x {SM_MAX_MHZ:.0f} MHz"}
+    for name, kind, iters in (("fp32_ffma", pp.PP_PROBE_FFMA, 1 << 16), ("tf32_mma", pp.PP_PROBE_MMA_TF32, 1 << 15),
+                              ("f16_mma", pp.PP_PROBE_MMA_F16, 1 << 15)):
+        pp.pp_peak_probe(kind, iters)  # warm-up (clocks ramp, code loads)
+        best = max((pp.pp_peak_probe(kind, iters) for _ in range(3)), key=lambda r: r[0])
+        out[name] = {"tflops": round(best[0], 2), "sm_mhz": round(best[1]), "ms": round(best[2], 3)}
+    return out
 
 
 def hbm_peak_gbs():
@@ -75,6 +100,9 @@ def workload(name: str):
         return synth.cfg2_style()
     if name == "vdsr":
         return synth.cfg3_vdsr()
+    if name.startswith("sweep:"):  # sweep:C:P:keep, one point of the throughput sweep
+        C, P, keep = name.split(":")[1:]
+        return synth.cfg4_point(int(C), int(P), float(keep))
     raise ValueError(name)
 
 
@@ -229,7 +257,7 @@ def time_net(dn, x, y, steps, warmup, flush, stream):
 
 
 def time_ops(dn, acts, steps, flush, stream):
-    """Average duration (ms) of every op's kernel launch, L2 flushed before each launch."""
+    """Average duration (ms) of every op's kernel launch alone, L2 flushed before each launch."""
     import torch
     from paper_2004_11250_gb300 import runner
     spec = dn.spec
@@ -253,6 +281,36 @@ def time_ops(dn, acts, steps, flush, stream):
     return res
 
 
+def time_ops_in_frame(dn, acts, steps, flush, stream):
+    """Median duration (ms) of every op inside a frame: the ops launched back to back in frame order on
+    the stream with a CUDA event between consecutive ops, L2 flushed once before each frame (as in the
+    timed frames).  The events break the overlap of one op's tail with the next op's start that the
+    frame's graph gets from programmatic dependent launch, so the sum is a little above the frame time."""
+    import torch
+    from paper_2004_11250_gb300 import runner
+    spec = dn.spec
+    n = len(spec.ops)
+    args = []
+    for k, (op, L) in enumerate(zip(spec.ops, dn.layers)):
+        xin = acts[k]
+        N, _, H, W = xin.shape
+        args.append((L, xin, acts[k + 1], acts[op.skip_from] if op.skip_from >= 0 else None, N, H, W,
+                     runner.op_flags(op)))
+    per = [[] for _ in range(n)]
+    for rep in range(steps + 2):
+        flush.zero_()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+        ev[0].record(stream)
+        for k, (L, xin, out, skip, N, H, W, flags) in enumerate(args):
+            L.forward(xin, out, skip, N, H, W, flags, stream)
+            ev[k + 1].record(stream)
+        ev[-1].synchronize()
+        if rep >= 2:  # two warm frames first
+            for k in range(n):
+                per[k].append(ev[k].elapsed_time(ev[k + 1]))
+    return [statistics.median(v) for v in per]
+
+
 def traffic_from_profile(kernel_hash: str, kernel: str = None):
     """Per-launch DRAM bytes (read + write) from the committed ncu summary of the VGG-16 frame, of one
     kernel (average over its launches in the frame) or of all the frame's convs, if that summary was
@@ -272,14 +330,6 @@ def traffic_from_profile(kernel_hash: str, kernel: str = None):
         return None
 
 
-def bf16_peak_tflops():
-    try:
-        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            return float(json.load(f)["bf16_tflops"]), "measured"
-    except Exception:
-        return BF16_PEAK_TFLOPS_FALLBACK, "fallback"
-
-
 def kernel_source_hash():
     """sha256 over the conv kernel sources (a profile taken on other sources is stale)."""
     import hashlib
@@ -290,24 +340,29 @@ def kernel_source_hash():
     return h.hexdigest()
 
 
+TENSOR_PEAKS = {}  # filled by main(): {"tf32": TFLOP/s, "f16": TFLOP/s} measured by pp_peak_probe
+
+
 def tensor_view(shapes, kern, op_ms, pruned):
     """Tensor-pipe view of the pruned ops that run on a tensor-core kernel: their dense 9-tap contraction
-    in 3 tf32 passes (hi*hi, lo*hi, hi*lo) per second against the tf32 peak; None without such ops."""
+    in 3 tf32 passes (hi*hi, lo*hi, hi*lo) per second against the measured kind::tf32 MMA peak; None
+    without such ops."""
     tc_ops = [k for k in pruned if kern[k] in ("ppconv_tc_kernel", "ppconv_tcf_kernel")]
-    if not tc_ops:
+    if not tc_ops or "tf32" not in TENSOR_PEAKS:
         return None
     tf = sum(3 * 2 * shapes[k]["N"] * shapes[k]["Ci"] * shapes[k]["Co"] * 9 * shapes[k]["H"] * shapes[k]["W"]
              for k in tc_ops)
     tt = sum(op_ms[k] for k in tc_ops) * 1e-3
-    bpk, bsrc = bf16_peak_tflops()
-    tpk = bpk * TF32_PER_BF16
+    tpk = TENSOR_PEAKS["tf32"]
     return {"bound": "tensor", "ops": len(tc_ops), "achieved": round(tf / tt / 1e12, 2), "peak": round(tpk, 1),
             "unit": "TFLOP/s (tf32, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
-            "peak_source": f"{bsrc} bf16 {bpk} TFLOP/s x nominal tf32/bf16 {TF32_PER_BF16:.3f}"}
+            "peak_source": "measured: pp_peak_probe kind::tf32 MMA (M 128, N 256, K 8), this run"}
 
 
-def bench_config(name, steps, warmup, flush, stream, hbm):
-    """ms/frame, GFLOP/s and per-op roofline fractions of one workload (used for the all-configs table)."""
+def bench_config(name, steps, warmup, flush, stream, hbm, fold_too=False):
+    """ms/frame, GFLOP/s and per-op roofline fractions (op times taken inside the frame) of one workload,
+    for the all-configs table; with fold_too also the frame time with the filter reorder folded into the
+    next layer (Section 3 matrix reorder; activations between layers in reordered channel order)."""
     import torch
     from paper_2004_11250_gb300 import runner
     spec = workload(name)
@@ -318,7 +373,7 @@ def bench_config(name, steps, warmup, flush, stream, hbm):
         ts = time_net(dn, x, y, steps, warmup, flush, stream)
         shapes = op_shapes(spec)
         acts = dn.run_layerwise(x)
-        op_ms = time_ops(dn, acts, max(3, steps // 2), flush, stream)
+        op_ms = time_ops_in_frame(dn, acts, max(3, steps // 2), flush, stream)
         flops = sum(s["flops"] for s in shapes)
         ms = statistics.median(ts)
         fr = [roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3) for s, t in zip(shapes, op_ms)]
@@ -328,12 +383,23 @@ def bench_config(name, steps, warmup, flush, stream, hbm):
         per_op = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "dense" for L in dn.layers]
         kern = sorted(set(k for k in per_op if k != "dense"))
         tv = tensor_view(shapes, per_op, op_ms, [k for k, s in enumerate(shapes) if s["pruned"]])
-        return {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1), "kernels": kern,
-                "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
-                "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None,
-                "tensor_tflops": tv["achieved"] if tv else None, "tensor_frac": tv["frac"] if tv else None}
+        res = {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1), "kernels": kern,
+               "op_us_in_frame": [round(t * 1e3, 2) for t in op_ms],
+               "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
+               "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None,
+               "tensor_tflops": tv["achieved"] if tv else None, "tensor_frac": tv["frac"] if tv else None}
     finally:
         dn.close()
+    if fold_too:
+        dn = runner.DeviceNet(spec, use_graph=True, fold_perm=True)
+        try:
+            x = torch.from_numpy(spec.x).cuda()
+            y = torch.empty(dn.out_shape, device="cuda")
+            ts = time_net(dn, x, y, steps, warmup, flush, stream)
+            res["ms_per_frame_perm_folded"] = round(statistics.median(ts), 4)
+        finally:
+            dn.close()
+    return res
 
 
 def bench_sweep(steps, flush, stream, hbm):
@@ -438,7 +504,12 @@ def metric_name(w):
              "single": "single pattern-pruned layer 1x16x32x32",
              "style": "style-transfer residual trunk 1x128x128x128",
              "vdsr": "VDSR-shaped SR stack 1x1x720x1280"}
-    return f"effective GFLOP/s (surviving MACs), {names[w]}, fp32"
+    if w.startswith("sweep:"):
+        C, P, keep = w.split(":")[1:]
+        name = f"sweep point 8x{C}x56x56, C_in = C_out = {C}, {P} patterns, keep {keep}"
+    else:
+        name = names[w]
+    return f"effective GFLOP/s (surviving MACs), {name}, fp32"
 
 
 def config_dict(w):
@@ -447,7 +518,9 @@ def config_dict(w):
     return {"workload": metric_name(w).split(", ")[1], "batch": int(spec.x.shape[0]),
             "input": list(spec.x.shape), "convs": len(spec.ops),
             "surviving_gflop_per_frame": round(spec.surviving_flops() / 1e9, 4),
-            "patterns": "8 fixed centre+3-neighbour patterns", "l2": "flushed between steps (512 MiB write)"}
+            "patterns": (f"{w.split(':')[2]} seed-chosen centre+3-neighbour patterns" if w.startswith("sweep:")
+                         else "8 fixed centre+3-neighbour patterns"),
+            "l2": "flushed between steps (512 MiB write)"}
 
 
 def main():
@@ -456,7 +529,10 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="vgg16", choices=["vgg16", "single", "style", "vdsr"])
+    ap.add_argument("--workload", default="vgg16",
+                    help="vgg16 (default), single, style, vdsr, or sweep:C:P:keep (one point of the sweep)")
+    ap.add_argument("--fold-perm", action="store_true",
+                    help="fold each layer's filter reorder into the next layer for the timed frames")
     ap.add_argument("--no-configs", action="store_true", help="skip the all-configs table")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -480,10 +556,15 @@ def main():
     stream = torch.cuda.Stream()
     torch.cuda.set_stream(stream)  # flushes, copies and kernels all ordered on one stream
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    # measured peaks of this GPU (the roofline denominators), before anything is timed
+    peaks = measure_peaks()
+    set_fp32_peak(peaks["fp32_ffma"]["tflops"])
+    TENSOR_PEAKS["tf32"] = peaks["tf32_mma"]["tflops"]
+    TENSOR_PEAKS["f16"] = peaks["f16_mma"]["tflops"]
     spec = workload(args.workload)
     shapes = op_shapes(spec)
     flops_frame = sum(s["flops"] for s in shapes)
-    dn = runner.DeviceNet(spec, use_graph=True)
+    dn = runner.DeviceNet(spec, use_graph=True, fold_perm=args.fold_perm)
     if args.kernels:
         from paper_2004_11250_gb300 import ppconv as pp
         ids = {"tm": pp.PP_KERNEL_TMEM, "reg": pp.PP_KERNEL_REGISTER, "tc": pp.PP_KERNEL_TC,
@@ -516,10 +597,13 @@ def main():
     ms_per_step = t_total_ms / args.steps
     value = job_value(ws, flops_frame, args.steps, t_total_ms)
 
-    # per-op kernel durations (same stream, L2 flushed before each launch) -> roofline of the pruned conv
+    # per-op kernel durations inside the frame (op by op in frame order, events between the ops, L2 flushed
+    # once per frame) -> roofline of the pruned convs; the same ops launched alone (L2 flushed before each
+    # launch) are reported beside them
     acts = dn.run_layerwise(x, stream)
     torch.cuda.synchronize()
-    op_ms = time_ops(dn, acts, max(5, args.steps // 2), flush, stream)
+    op_ms = time_ops_in_frame(dn, acts, max(5, args.steps // 2), flush, stream)
+    op_ms_alone = time_ops(dn, acts, max(5, args.steps // 2), flush, stream)
     del acts
     pruned = [k for k, s in enumerate(shapes) if s["pruned"]]
     kf = sum(shapes[k]["flops"] for k in pruned)
@@ -547,6 +631,7 @@ def main():
     dom = max(by_kern, key=lambda n: by_kern[n][1])
     dom_ops = [k for k in pruned if kern[k] == dom]
     achieved = by_kern[dom][0] / by_kern[dom][1] / 1e12
+    achieved_alone = sum(shapes[k]["flops"] for k in dom_ops) / (sum(op_ms_alone[k] for k in dom_ops) * 1e-3) / 1e12
     traffic = traffic_from_profile(kernel_source_hash(), dom)
     layer_fracs = [round(roof_time_s(s["flops"], s["bytes"], hbm) / (t * 1e-3), 3) for s, t in zip(shapes, op_ms)]
 
@@ -568,7 +653,7 @@ def main():
     if not args.no_configs and rank == 0:
         configs = {}
         for name in ("single", "vgg16", "style", "vdsr"):
-            configs[name] = bench_config(name, 10, 3, flush, stream, hbm)
+            configs[name] = bench_config(name, 10, 3, flush, stream, hbm, fold_too=name in ("vgg16", "style"))
         configs["sweep"] = bench_sweep(5, flush, stream, hbm)
 
     cpu = None
@@ -599,20 +684,32 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded; shapes and distributions of the workload, no dataset or trained weights)",
-            "config": config_dict(args.workload),
+            "config": dict(config_dict(args.workload), perm_folded=bool(args.fold_perm)),
             "e2e": {"value": round(e2e_value, 2), "unit": "GFLOP/s", "h2d_bytes_per_step": int(xh.numel() * 4),
                     "d2h_bytes_per_step": int(yh.numel() * 4), "ms_per_step": round(statistics.median(e2e_t) * 1e3, 4)},
             "gpu_launches": len(spec.ops) * args.steps,
             "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
                          "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
                          "kernel": f"{dom} ({len(dom_ops)} of the {len(pruned)} pruned convs, "
-                                   f"{100 * by_kern[dom][1] / kt:.0f}% of their device time)",
+                                   f"{100 * by_kern[dom][1] / kt:.0f}% of their in-frame device time)",
+                         "timing": "op by op in frame order, CUDA events between the ops on the launching "
+                                   "stream, L2 flushed once per frame; median over frames",
+                         "op_us_in_frame": [round(t * 1e3, 2) for t in op_ms],
+                         "op_flops": [int(s["flops"]) for s in shapes],
+                         "dominant_ops": dom_ops,
+                         "frame_ms_op_by_op": round(sum(op_ms), 4),
+                         "alone": {"achieved": round(achieved_alone, 3),
+                                   "frac": round(achieved_alone / FP32_PEAK_TFLOPS, 4),
+                                   "op_us": [round(t * 1e3, 2) for t in op_ms_alone],
+                                   "timing": "each op launched alone, L2 flushed before every launch"},
                          "all_pruned_ops": {"achieved": round(achieved_all, 3),
                                             "frac": round(achieved_all / FP32_PEAK_TFLOPS, 4),
                                             "traffic": traffic_from_profile(kernel_source_hash()),
                                             "kernels": sorted(by_kern)},
                          "tensor": tensor,
-                         "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
+                         "peak_source": (f"measured: pp_peak_probe FFMA, {peaks['fp32_ffma']['tflops']} TFLOP/s at "
+                                         f"{peaks['fp32_ffma']['sm_mhz']} MHz (this run)"),
+                         "peaks": peaks,
                          "hbm_peak_gbs": hbm, "hbm_peak_source": hbm_src},
             "layer_roofline_frac": layer_fracs,
             "layer_kernels": kern,

@@ -115,6 +115,17 @@ pp_status pp_unpack_layer(const pp_packed* pk, float* w_out, uint8_t* mask_out);
 
 void pp_packed_destroy(pp_packed* pk);
 
+/* Permute the input channels of a layer's dense description, for packing a
+ * layer whose input activation is stored in another channel order (see
+ * pp_layer_set_output_order): position c of the result holds original input
+ * channel layout[c], i.e. w_out[o][c][t] = w[o][layout[c]][t], and likewise
+ * mask_out[o][c] and ids_out[o][c] (each optional: NULL skips it; its source
+ * must then be given only if its output is).  Host only; outputs must not
+ * overlap inputs.  Errors: PP_ERR_INVALID_ARG (null pointer, Co or Ci < 1,
+ * layout not a permutation of 0..Ci-1, an output without its input). */
+pp_status pp_permute_input_channels(const float* w, const uint8_t* mask, const uint8_t* pattern_ids, int Co, int Ci,
+                                    const int32_t* layout, float* w_out, uint8_t* mask_out, uint8_t* ids_out);
+
 /* Fold an inference batch normalisation that follows the convolution into its
  * weights and bias (Section 3: convolution fused with the layers after it), in
  * place on host arrays before packing: w [Co][Ci][9] becomes w * g[o] and
@@ -177,6 +188,24 @@ pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const
  */
 pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H,
                                   int W, int flags, void* stream);
+
+/*
+ * Output channel order of a layer (Section 3 "Matrix reorder", folded into
+ * the next layer).  order[o] = the output channel where original filter o is
+ * stored (a permutation of 0..Co-1, host array); NULL restores the original
+ * order (order[o] = o), the default.  Every kernel and pp_conv_forward_noalloc
+ * honour it; a skip tensor (PP_ADD_SKIP) is read at the same channel as the
+ * output it is added to.
+ * Folding the filter reorder of layer k into layer k + 1: give layer k
+ * order[perm_k[j]] = j (filter j of the reordered layer is stored at channel
+ * j, so the epilogue writes the filters in the order they are computed), and
+ * pack layer k + 1 from weights whose input channels were permuted the same
+ * way (pp_permute_input_channels with layout = perm_k).
+ * Synchronous on stream (uploads Co indices; layers with a direct-kernel
+ * layout also rebuild it).  A CUDA graph captured earlier keeps the direct
+ * kernel's old weights: re-capture after calling this (pp_net_use_graph).
+ * Errors: PP_ERR_INVALID_ARG (not a permutation), PP_ERR_CUDA, PP_ERR_OOM. */
+pp_status pp_layer_set_output_order(pp_layer* layer, const int32_t* order, void* stream);
 
 /* Which kernel pp_conv_forward runs for a layer.  All compute the same
  * convolution within the documented fp32 bound.
@@ -262,6 +291,33 @@ pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);
  * Errors: PP_ERR_INVALID_ARG (null pointer, polls out of range), PP_ERR_OOM,
  * PP_ERR_CUDA. */
 pp_status pp_wait_probe(long long polls, int* gave_up, long long* elapsed_ns);
+
+/* Peak-rate probes (diagnostics; the paper has no counterpart).  One launch
+ * keeps a single execution pipe busy on every SM of the current device and
+ * reports its rate, so roofline fractions can be taken against a measured
+ * peak instead of a data-sheet figure:
+ *   PP_PROBE_FFMA      fp32 fused multiply-add on the CUDA cores (16
+ *                      independent chains per thread, 4 CTAs of 256 threads
+ *                      per SM), 2 FLOP per multiply-add;
+ *   PP_PROBE_MMA_TF32  tcgen05.mma kind::tf32, M = 128, N = 256, K = 8 per
+ *                      instruction, one issuing thread per SM, operands in
+ *                      shared memory, accumulator in tensor memory;
+ *   PP_PROBE_MMA_F16   the same with kind::f16 (f16 operands, fp32
+ *                      accumulation), K = 16.
+ *   iters   multiply-add groups per thread (FFMA) or MMA instructions per SM,
+ *           1 .. 2^24; pick it so the launch takes a few milliseconds
+ *   tflops  FLOP of the launch / its duration (CUDA events), in TFLOP/s
+ *   sm_mhz  SM clock during the launch: SM cycles over the global timer of
+ *           one CTA, in MHz
+ *   ms      duration of the launch
+ * Synchronous, on the legacy default stream; allocates and frees a small
+ * result buffer.  Errors: PP_ERR_INVALID_ARG (null pointer, kind, iters out
+ * of range), PP_ERR_OOM, PP_ERR_CUDA (also when an MMA probe's bounded wait
+ * for its instructions ran out). */
+#define PP_PROBE_FFMA 0
+#define PP_PROBE_MMA_TF32 1
+#define PP_PROBE_MMA_F16 2
+pp_status pp_peak_probe(int kind, long long iters, double* tflops, double* sm_mhz, double* ms);
 
 void pp_layer_destroy(pp_layer* layer);
 

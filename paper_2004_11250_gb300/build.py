@@ -17,7 +17,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libppconv.so")
 
-SOURCES = ["pack.cpp", "conv.cu", "conv_tm.cu", "conv_tc.cu", "conv_tcf.cu", "conv_direct.cu", "net.cpp"]
+SOURCES = ["pack.cpp", "conv.cu", "conv_tm.cu", "conv_tc.cu", "conv_tcf.cu", "conv_direct.cu", "probe.cu", "net.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-I" + INCLUDE, "-I" + CSRC, "-Xcompiler", "-fPIC,-O3"]
 

@@ -410,8 +410,11 @@ struct pp_layer {
   int* cofs = nullptr;
   uint32_t* code = nullptr;
   float4* wts = nullptr;
-  int* perm = nullptr;
+  int* perm = nullptr;   // [Co] output channel of reordered filter j (the packer's perm unless re-ordered)
   float* bias = nullptr;
+  std::vector<int32_t> pk_perm;     // the packer's filter permutation (host copy)
+  std::vector<float> direct_w;      // direct layout's dense weights [Co][Ci][9], original filter order
+  std::vector<float> direct_bias;   // and its bias (empty: none)
 };
 
 struct pp_dense {
@@ -524,24 +527,21 @@ cudaError_t set_attributes() {
 }
 
 // Once per process and device: allow the kernels' dynamic shared memory.
+ppc::DeviceOnce g_kernels_once;
 cudaError_t prepare_kernels() {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  static bool done[64] = {};
-  if (dev < 64 && done[dev]) return cudaSuccess;
-  if ((e = set_attributes<MODE_RING8, false>()) != cudaSuccess) return e;
-  if ((e = set_attributes<MODE_RING8, true>()) != cudaSuccess) return e;
-  if ((e = set_attributes<MODE_GENERIC, false>()) != cudaSuccess) return e;
-  if ((e = set_attributes<MODE_GENERIC, true>()) != cudaSuccess) return e;
-  if (dev < 64) done[dev] = true;
-  return cudaSuccess;
+  return g_kernels_once.run([](int) {
+    cudaError_t e;
+    if ((e = set_attributes<MODE_RING8, false>()) != cudaSuccess) return e;
+    if ((e = set_attributes<MODE_RING8, true>()) != cudaSuccess) return e;
+    if ((e = set_attributes<MODE_GENERIC, false>()) != cudaSuccess) return e;
+    return set_attributes<MODE_GENERIC, true>();
+  });
 }
 
 // Number of CTAs sharing one output tile: split the input chunks over a
 // cluster when the grid alone would leave SMs idle (two CTAs fit per SM).
 int choose_split(int64_t base_ctas, int nch) {
-  int sms = 152;
+  const int sms = ppc::device_sms();
   int ks = 1;
   while (ks < MAX_SPLIT && ks * 2 <= nch && base_ctas * ks < 2 * sms) ks *= 2;
   return ks;
@@ -598,11 +598,11 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
   p.flags = flags;
   const int cgroups = (L->G + NWF - 1) / NWF;
   const int64_t base = (int64_t)tiles_y * tiles_x * cgroups * N;
+  if (prepare_kernels() != cudaSuccess || ppc::device_sms() <= 0) return PP_ERR_CUDA;
   const int ks = choose_split(base, L->nch);
   p.ksplit = ks;
   p.cpk = (L->nch + ks - 1) / ks;
   if ((int64_t)N * ks > 65535 || cgroups > 65535) return PP_ERR_UNSUPPORTED;
-  if (prepare_kernels() != cudaSuccess) return PP_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(tiles_y * tiles_x, cgroups, N * ks);
   cfg.blockDim = dim3(NTHREADS);
@@ -631,6 +631,21 @@ pp_status launch(const pp_layer* L, const float* x, float* y, const float* skip,
 }
 
 }  // namespace
+
+namespace ppc {
+
+int device_sms() {
+  static DeviceOnce once;
+  static int sms[DeviceOnce::kMaxDevices];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= DeviceOnce::kMaxDevices) return 0;
+  if (once.run([](int d) { return cudaDeviceGetAttribute(&sms[d], cudaDevAttrMultiProcessorCount, d); }) !=
+      cudaSuccess)
+    return 0;
+  return sms[dev];
+}
+
+}  // namespace ppc
 
 extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, void* stream, pp_layer** out) {
   if (!pk || !out) return PP_ERR_INVALID_ARG;
@@ -683,11 +698,14 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
           wd[((size_t)pk->perm[j] * pk->Ci + pk->kidx[e]) * 9 + t[s]] = pk->kw[(size_t)e * 4 + s];
       }
     st = ppc::direct_build(&L->direct, wd.data(), bias, pk->Co, pk->Ci, (cudaStream_t)stream);
+    L->direct_w.swap(wd);
+    if (bias) L->direct_bias.assign(bias, bias + pk->Co);
   }
   if (st != PP_OK) {
     pp_layer_destroy(L);
     return st;
   }
+  L->pk_perm = pk->perm;
   // Kernel choice by estimated SM cycles per pixel: the tensor cores run the
   // dense 9-tap contraction (filters padded to 128, channels to 8) three times
   // at ~1800 multiply-adds per cycle; the FMA kernels run only the kept taps
@@ -702,6 +720,41 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
   if (L->direct.w && pk->Ci <= 4) L->auto_kernel = PP_KERNEL_DIRECT;
   L->kernel = L->auto_kernel;
   *out = L;
+  return PP_OK;
+}
+
+extern "C" pp_status pp_layer_set_output_order(pp_layer* L, const int32_t* order, void* stream_) {
+  if (!L) return PP_ERR_INVALID_ARG;
+  const int Co = L->Co, Ci = L->Ci;
+  std::vector<int32_t> ord(Co);
+  std::vector<uint8_t> seen(Co, 0);
+  for (int o = 0; o < Co; ++o) {
+    ord[o] = order ? order[o] : o;
+    if (ord[o] < 0 || ord[o] >= Co || seen[ord[o]]) return PP_ERR_INVALID_ARG;
+    seen[ord[o]] = 1;
+  }
+  cudaStream_t stream = (cudaStream_t)stream_;
+  // every kernel but the direct one stores reordered filter j at channel perm[j]
+  std::vector<int32_t> store(Co);
+  for (int j = 0; j < Co; ++j) store[j] = ord[L->pk_perm[j]];
+  if (cudaMemcpyAsync(L->perm, store.data(), (size_t)Co * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess) {
+    cudaGetLastError();
+    return PP_ERR_CUDA;
+  }
+  if (L->direct.w) {
+    // the direct kernel stores row o of its dense weights at channel o: rebuild them with rows moved
+    std::vector<float> w((size_t)Co * Ci * 9), b(L->direct_bias.empty() ? 0 : Co);
+    for (int o = 0; o < Co; ++o) {
+      std::memcpy(&w[(size_t)ord[o] * Ci * 9], &L->direct_w[(size_t)o * Ci * 9], (size_t)Ci * 9 * sizeof(float));
+      if (!b.empty()) b[ord[o]] = L->direct_bias[o];
+    }
+    ppc::DirectLayout D;
+    const pp_status st = ppc::direct_build(&D, w.data(), b.empty() ? nullptr : b.data(), Co, Ci, stream);
+    if (st != PP_OK) return st;
+    ppc::direct_free(&L->direct);
+    L->direct = D;
+  }
   return PP_OK;
 }
 

@@ -190,15 +190,11 @@ __global__ void __launch_bounds__(DTHREADS, FBD >= 16 ? 2 : 3) ppconv_direct_ker
 template <int CC, int FBD>
 cudaError_t launch_one(const DirectParams& p, dim3 grid, cudaStream_t stream) {
   constexpr int bytes = 2 * (CC * DTW * DPITCH + CC * FBD * 12) * 4;
-  static bool attr_set[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!attr_set[dev]) {
-    const cudaError_t e =
-        cudaFuncSetAttribute(ppconv_direct_kernel<CC, FBD>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e != cudaSuccess) return e;
-    attr_set[dev] = true;
-  }
+  static ppc::DeviceOnce attr_once;  // one per instantiation
+  const cudaError_t ea = attr_once.run([](int) {
+    return cudaFuncSetAttribute(ppconv_direct_kernel<CC, FBD>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  });
+  if (ea != cudaSuccess) return ea;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -594,41 +594,41 @@ cudaError_t set_attr() {
                               Geo<ORI, TW, FB>::SMEM_ALLOC);
 }
 
-bool g_done[64] = {};
+ppc::DeviceOnce g_attr_once;
 
 cudaError_t prepare() {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 64 && g_done[dev]) return cudaSuccess;
-  if ((e = set_attr<ORI_FP, 16, 128>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_FP, 32, 128>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_FP, 64, 128>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_FP, 128, 128>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_PF, 128, 64>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_PF, 128, 128>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_PFR, 16, 64>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_PFR, 32, 64>()) != cudaSuccess) return e;
-  if ((e = set_attr<ORI_PFR, 64, 64>()) != cudaSuccess) return e;
-  if (dev < 64) g_done[dev] = true;
-  return cudaSuccess;
+  return g_attr_once.run([](int) {
+    cudaError_t e;
+    if ((e = set_attr<ORI_FP, 16, 128>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_FP, 32, 128>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_FP, 64, 128>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_FP, 128, 128>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_PF, 128, 64>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_PF, 128, 128>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_PFR, 16, 64>()) != cudaSuccess) return e;
+    if ((e = set_attr<ORI_PFR, 32, 64>()) != cudaSuccess) return e;
+    return set_attr<ORI_PFR, 64, 64>();
+  });
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-EncodeTiledFn g_encode = nullptr;
+// cuTensorMapEncodeTiled from the driver (null: every launch uses per-thread loads)
+std::atomic<EncodeTiledFn> g_encode{nullptr};
+ppc::DeviceOnce g_encode_once;
 
 // 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][8][R+2][TW+8].
 template <int ORI, int TW, int FB>
 bool make_xmap(CUtensorMap* m, const TcParams& p) {
   using G = Geo<ORI, TW, FB>;
-  if (!g_encode) return false;
+  const EncodeTiledFn encode = g_encode.load(std::memory_order_acquire);
+  if (!encode) return false;
   const cuuint64_t dims[4] = {(cuuint64_t)p.W, (cuuint64_t)p.H, (cuuint64_t)p.Ci, (cuuint64_t)p.N};
   const cuuint64_t strides[3] = {(cuuint64_t)p.W * 4, (cuuint64_t)p.W * p.H * 4, (cuuint64_t)p.W * p.H * p.Ci * 4};
   const cuuint32_t box[4] = {(cuuint32_t)G::RAW_W, (cuuint32_t)G::BROWS, (cuuint32_t)KC, 1};
   const cuuint32_t estr[4] = {1, 1, 1, 1};
-  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(p.x), dims, strides, box, estr,
+  return encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(p.x), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -660,29 +660,24 @@ cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
   return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB>, p, xmap);
 }
 
-int g_sms = 0;
-
 }  // namespace
 
 namespace ppc {
 
 pp_status tc_prepare() {
-  if (prepare() != cudaSuccess) return PP_ERR_CUDA;
-  if (!g_encode) {
+  if (prepare() != cudaSuccess || device_sms() <= 0) return PP_ERR_CUDA;
+  // the entry point is process-wide; looked up at the first set-up of each device
+  const cudaError_t e = g_encode_once.run([](int) {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+      g_encode.store(reinterpret_cast<EncodeTiledFn>(fn), std::memory_order_release);
     else
       cudaGetLastError();  // without the entry point every launch uses per-thread loads
-  }
-  if (!g_sms) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-      return PP_ERR_CUDA;
-  }
-  return PP_OK;
+    return cudaSuccess;
+  });
+  return e == cudaSuccess ? PP_OK : PP_ERR_CUDA;
 }
 
 // Dense per-tap weights of every (FB-filter block, 8-channel chunk), split into
@@ -787,20 +782,21 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
   p.flags = flags;
   int ori, tw;
   tc_geometry(T, W, (flags & PP_POOL2) != 0, &ori, &tw);
+  const int sms = device_sms();
   cudaError_t e;
   if (ori == ORI_PF)
-    e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, g_sms) : launch<ORI_PF, 128, 128>(p, stream, g_sms);
+    e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, sms) : launch<ORI_PF, 128, 128>(p, stream, sms);
   else if (ori == ORI_PFR)
-    e = tw == 16 ? launch<ORI_PFR, 16, 64>(p, stream, g_sms)
-                 : tw == 32 ? launch<ORI_PFR, 32, 64>(p, stream, g_sms) : launch<ORI_PFR, 64, 64>(p, stream, g_sms);
+    e = tw == 16 ? launch<ORI_PFR, 16, 64>(p, stream, sms)
+                 : tw == 32 ? launch<ORI_PFR, 32, 64>(p, stream, sms) : launch<ORI_PFR, 64, 64>(p, stream, sms);
   else if (tw == 16)
-    e = launch<ORI_FP, 16, 128>(p, stream, g_sms);
+    e = launch<ORI_FP, 16, 128>(p, stream, sms);
   else if (tw == 32)
-    e = launch<ORI_FP, 32, 128>(p, stream, g_sms);
+    e = launch<ORI_FP, 32, 128>(p, stream, sms);
   else if (tw == 64)
-    e = launch<ORI_FP, 64, 128>(p, stream, g_sms);
+    e = launch<ORI_FP, 64, 128>(p, stream, sms);
   else
-    e = launch<ORI_FP, 128, 128>(p, stream, g_sms);
+    e = launch<ORI_FP, 128, 128>(p, stream, sms);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return PP_ERR_CUDA;

@@ -606,24 +606,22 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 struct DeviceState {
-  bool ready = false;
   int sms = 0;
   int max_clusters[MAX_SPLIT + 1] = {};  // co-resident clusters of each size (0: size unusable)
   EncodeTiledFn encode = nullptr;
 };
-DeviceState g_dev[64];
+DeviceState g_dev[ppc::DeviceOnce::kMaxDevices];
+ppc::DeviceOnce g_dev_once;  // fills g_dev[dev] once per device (its ready flag publishes it)
 
-DeviceState* prepare() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+cudaError_t init_device(int dev) {
   DeviceState& D = g_dev[dev];
-  if (D.ready) return &D;
-  if (cudaDeviceGetAttribute(&D.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return nullptr;
-  if (cudaFuncSetAttribute(ppconv_tcf_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
+  cudaError_t e = cudaDeviceGetAttribute(&D.sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(ppconv_tcf_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
           cudaSuccess ||
-      cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC) !=
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
           cudaSuccess)
-    return nullptr;
+    return e;
   if (cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
     cudaGetLastError();  // then only portable sizes (up to 8) can be used
   for (int s = 2; s <= MAX_SPLIT; s *= 2) {
@@ -652,8 +650,15 @@ DeviceState* prepare() {
     D.encode = reinterpret_cast<EncodeTiledFn>(fn);
   else
     cudaGetLastError();  // without the entry point every launch uses per-thread loads
-  D.ready = true;
-  return &D;
+  return cudaSuccess;
+}
+
+// The current device's state, set up on first use (thread-safe), or null.
+DeviceState* prepare() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= ppc::DeviceOnce::kMaxDevices) return nullptr;
+  if (g_dev_once.run(init_device) != cudaSuccess) return nullptr;
+  return &g_dev[dev];
 }
 
 struct FlatGeo {

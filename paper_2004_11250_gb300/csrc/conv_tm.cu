@@ -430,21 +430,16 @@ int choose_split(int64_t base_ctas, int nch) {
   return best;
 }
 
-bool g_attr_done[64] = {};
+
+ppc::DeviceOnce g_attr_once;
 
 cudaError_t prepare() {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 64 && g_attr_done[dev]) return cudaSuccess;
-  if ((e = cudaFuncSetAttribute(ppconv_tm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES)) !=
-      cudaSuccess)
-    return e;
-  if ((e = cudaFuncSetAttribute(ppconv_tm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES)) !=
-      cudaSuccess)
-    return e;
-  if (dev < 64) g_attr_done[dev] = true;
-  return cudaSuccess;
+  return g_attr_once.run([](int) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(ppconv_tm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(ppconv_tm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  });
 }
 
 }  // namespace

@@ -3,7 +3,9 @@
 
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
+#include <mutex>
 #include <vector>
 
 #include "ppconv.h"
@@ -22,6 +24,33 @@ struct pp_packed {
 };
 
 namespace ppc {
+
+// Once-per-device set-up of a launch path (kernel attributes, device queries).
+// run(init) calls init(dev) with the current device `dev` until one call
+// succeeds; concurrent first calls from several host threads serialise on the
+// mutex, and a caller that finds the ready flag set (acquire) sees everything
+// the successful init wrote (release).  A failed init is retried next time.
+struct DeviceOnce {
+  static constexpr int kMaxDevices = 64;
+  std::mutex mu;
+  std::atomic<bool> ready[kMaxDevices]{};
+  template <class F>
+  cudaError_t run(F&& init) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    if (ready[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    std::lock_guard<std::mutex> lock(mu);
+    if (ready[dev].load(std::memory_order_relaxed)) return cudaSuccess;
+    e = init(dev);
+    if (e == cudaSuccess) ready[dev].store(true, std::memory_order_release);
+    return e;
+  }
+};
+
+// Number of SMs of the current device (queried once per device).
+int device_sms();
 
 // Maximum filter slots handled by one warp of the conv kernel.
 constexpr int kSlots = 16;

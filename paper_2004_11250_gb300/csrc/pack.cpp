@@ -217,6 +217,27 @@ extern "C" pp_status pp_fold_batchnorm(float* w, float* bias, const float* gamma
   return PP_OK;
 }
 
+extern "C" pp_status pp_permute_input_channels(const float* w, const uint8_t* mask, const uint8_t* pattern_ids,
+                                               int Co, int Ci, const int32_t* layout, float* w_out,
+                                               uint8_t* mask_out, uint8_t* ids_out) {
+  if (!w || !layout || !w_out || Co < 1 || Ci < 1) return PP_ERR_INVALID_ARG;
+  if ((mask_out && !mask) || (ids_out && !pattern_ids)) return PP_ERR_INVALID_ARG;
+  std::vector<uint8_t> seen(Ci, 0);
+  for (int c = 0; c < Ci; ++c) {
+    if (layout[c] < 0 || layout[c] >= Ci || seen[layout[c]]) return PP_ERR_INVALID_ARG;
+    seen[layout[c]] = 1;
+  }
+  // position c of the permuted layer reads original input channel layout[c]
+  for (int o = 0; o < Co; ++o)
+    for (int c = 0; c < Ci; ++c) {
+      const size_t src = size_t(o) * Ci + layout[c], dst = size_t(o) * Ci + c;
+      std::memcpy(w_out + dst * 9, w + src * 9, 9 * sizeof(float));
+      if (mask_out) mask_out[dst] = mask[src];
+      if (ids_out) ids_out[dst] = pattern_ids[src];
+    }
+  return PP_OK;
+}
+
 extern "C" const char* pp_status_string(pp_status s) {
   switch (s) {
     case PP_OK: return "PP_OK";

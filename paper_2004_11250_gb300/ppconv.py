@@ -42,6 +42,10 @@ PP_KERNEL_DIRECT = 5
 
 PP_WAIT_POLLS = 1 << 18
 
+PP_PROBE_FFMA = 0
+PP_PROBE_MMA_TF32 = 1
+PP_PROBE_MMA_F16 = 2
+
 PP_ADD_SKIP = 1
 PP_RELU = 2
 PP_POOL2 = 4
@@ -65,9 +69,12 @@ _SIGS = {
     "pp_conv_forward": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
     "pp_conv_forward_noalloc": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
     "pp_layer_set_kernel": ([_P, _I], _I),
+    "pp_layer_set_output_order": ([_P, _P, _P], _I),
+    "pp_permute_input_channels": ([_P, _P, _P, _I, _I, _P, _P, _P, _P], _I),
     "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_device_status": ([_P, _P], _I),
     "pp_wait_probe": ([ctypes.c_longlong, _P, _P], _I),
+    "pp_peak_probe": ([_I, ctypes.c_longlong, _P, _P, _P], _I),
     "pp_layer_autotune": ([_P, _I, _I, _I, _I, _P], _I),
     "pp_layer_flat_geometry": ([_P, _I, _I, _I, _I, _P, _P], _I),
     "pp_layer_pin_flat_geometry": ([_P, _I, _I, _I, _I, _I, _I], _I),
@@ -112,6 +119,24 @@ def pp_fold_batchnorm(w, bias, gamma, beta, mean, var, eps=1e-5):
     _check(lib.pp_fold_batchnorm(w2.ctypes.data, b2.ctypes.data, *[a.ctypes.data for a in arrs], float(eps), Co, Ci),
            "pp_fold_batchnorm")
     return w2, b2
+
+
+def pp_permute_input_channels(w, mask, layout, pattern_ids=None):
+    """(w, mask, ids) with input channel c of the result = original channel layout[c]; ids None if not given."""
+    w = _host(w, np.float32)
+    Co, Ci = w.shape[0], w.shape[1]
+    w = w.reshape(Co, Ci, 9)
+    mask = _host(mask, np.uint8)
+    ids = _host(pattern_ids, np.uint8)
+    lay = _host(layout, np.int32)
+    if mask.shape != (Co, Ci) or lay.shape != (Ci,) or (ids is not None and ids.shape != (Co, Ci)):
+        raise PPError(PP_ERR_INVALID_ARG, "pp_permute_input_channels shapes")
+    w2 = np.empty_like(w)
+    m2 = np.empty_like(mask)
+    i2 = None if ids is None else np.empty_like(ids)
+    _check(lib.pp_permute_input_channels(_hp(w), _hp(mask), _hp(ids), Co, Ci, _hp(lay), _hp(w2), _hp(m2), _hp(i2)),
+           "pp_permute_input_channels")
+    return w2, m2, i2
 
 
 def pp_status_string(code: int) -> str:
@@ -243,6 +268,12 @@ def pp_layer_set_kernel(layer, kernel: int):
     _check(lib.pp_layer_set_kernel(layer, kernel), "pp_layer_set_kernel")
 
 
+def pp_layer_set_output_order(layer, order=None, stream=None):
+    """order[o] = output channel of original filter o (None: original order); see the header."""
+    o = _host(order, np.int32)
+    _check(lib.pp_layer_set_output_order(layer, _hp(o), _stream(stream)), "pp_layer_set_output_order")
+
+
 def pp_layer_kernel(layer) -> int:
     k = _I()
     _check(lib.pp_layer_kernel(layer, ctypes.byref(k)), "pp_layer_kernel")
@@ -275,6 +306,13 @@ def pp_wait_probe(polls: int):
     g, ns = _I(), ctypes.c_longlong()
     _check(lib.pp_wait_probe(polls, ctypes.byref(g), ctypes.byref(ns)), "pp_wait_probe")
     return g.value, ns.value
+
+
+def pp_peak_probe(kind: int, iters: int):
+    """(TFLOP/s, SM MHz, ms) of one launch of a peak-rate probe (PP_PROBE_*; see the header)."""
+    tf, mhz, ms = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    _check(lib.pp_peak_probe(kind, iters, ctypes.byref(tf), ctypes.byref(mhz), ctypes.byref(ms)), "pp_peak_probe")
+    return tf.value, mhz.value, ms.value
 
 
 def pp_layer_destroy(layer):

@@ -182,3 +182,59 @@ def test_wait_probe_rejects_bad_arguments(pp):
         with pytest.raises(pp.PPError) as e:
             pp.pp_wait_probe(polls)
         assert e.value.code == pp.PP_ERR_INVALID_ARG
+
+
+def test_peak_probe_rejects_bad_arguments(pp):
+    """Argument checks come before any device work (this runs without a GPU)."""
+    for kind, iters in ((pp.PP_PROBE_FFMA, 0), (pp.PP_PROBE_MMA_TF32, (1 << 24) + 1), (7, 100), (-1, 100)):
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_peak_probe(kind, iters)
+        assert e.value.code == pp.PP_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("idx", [0, 1, 2, 6])
+def test_permuted_input_channels_pack_matches_oracle(pp, oracle_mod, idx):
+    """Folding the filter reorder of one layer into the next (Section 3 "Matrix reorder"): the next
+    layer's input channels are permuted on the host before packing.  pp_permute_input_channels equals
+    numpy fancy indexing bit for bit, and the packed metadata of the permuted layer equals the oracle's
+    packing of the numpy-permuted layer bit for bit."""
+    L = layers_for_pack()[idx]
+    rng = np.random.default_rng(100 + idx)
+    layout = rng.permutation(L.Ci).astype(np.int32)
+    w2, m2, i2 = pp.pp_permute_input_channels(L.w, L.mask, layout, L.pattern_ids)
+    wn = L.w.reshape(L.Co, L.Ci, 9)[:, layout]
+    assert (w2.view(np.uint32) == wn.view(np.uint32)).all()
+    assert (m2 == L.mask[:, layout]).all() and (i2 == L.pattern_ids[:, layout]).all()
+    ref = oracle_mod.pack(wn, L.mask[:, layout], L.taps)
+    pk = pp.pp_pack_layer(w2, m2, L.taps)
+    try:
+        a = pp.pp_packed_arrays(pk)
+        for k in ("perm", "kptr", "kidx", "kpat"):
+            assert (a[k] == getattr(ref, k)).all(), k
+        assert (a["kw"].view(np.uint32) == ref.kw.view(np.uint32)).all()
+    finally:
+        pp.pp_packed_destroy(pk)
+    # the identity layout is a no-op; a repeated channel is not a permutation
+    w3, _, _ = pp.pp_permute_input_channels(L.w, L.mask, np.arange(L.Ci, dtype=np.int32))
+    assert (w3.view(np.uint32) == L.w.reshape(L.Co, L.Ci, 9).view(np.uint32)).all()
+    if L.Ci > 1:
+        bad = layout.copy()
+        bad[0] = bad[1]
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_permute_input_channels(L.w, L.mask, bad)
+        assert e.value.code == pp.PP_ERR_INVALID_ARG
+
+
+def test_fold_groups_of_the_workloads():
+    """Host logic of the permutation folding: which activations keep the original channel order."""
+    from paper_2004_11250_gb300 import runner
+    g = runner.fold_groups(synth.cfg1_vgg16())
+    assert g[0] and g[-1] and not any(g[1:-1])
+    net = synth.cfg2_style()
+    g = runner.fold_groups(net)
+    # block inputs and outputs are tied to the network input through the skips; conv1 outputs are free
+    assert g == [True] + [op.skip_from >= 0 for op in net.ops]
+    net = synth.cfg3_vdsr(H=8, W=8)
+    g = runner.fold_groups(net)
+    # dense end layers and the global skip keep the original order, the 18 pruned layers' outputs are free
+    assert g[0] and g[1] and g[-1] and g[-2] is False and not any(g[2:-2])

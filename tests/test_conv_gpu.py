@@ -1,8 +1,8 @@
 """GPU parity: the CUDA path, called through the C-ABI, against the fp64 oracle.
 
-Small layers are compared on every output; the five workloads at full size are
-compared layer by layer (each layer's oracle runs on the GPU's own input to that
-layer) on sampled outputs including borders and tile edges.  Bound:
+Every output is compared: small layers, and the five workloads at full size
+layer by layer (each layer's oracle runs on the GPU's own input to that layer),
+including all 48 sweep points and the multi-tile repeatability shapes.  Bound:
 |gpu - oracle| <= 1e-5 * S per output (see tests/parity.py); integer-valued
 cases must be bit-exact.
 """
@@ -11,7 +11,7 @@ import pytest
 import torch
 
 from paper_2004_11250_gb300 import synth
-from parity import check_within, oracle_layer_full, oracle_layer_points, sample_points
+from parity import check_within, oracle_layer_full, to_original
 
 pytestmark = pytest.mark.gpu
 
@@ -265,7 +265,7 @@ def test_tensor_core_repeatable_multi_tile(pp, runner, oracle_mod, shape, kernel
     buffers wrap many times, or (flat kernel, few tiles) channel chunks split over
     clusters.  The kernels' summation order is fixed, so repeated
     runs must agree bit for bit (a pipeline race shows up as a run-to-run
-    difference); one run is also checked against the oracle on sampled outputs."""
+    difference); one run is also checked against the oracle on every output."""
     N, Ci, Co, H, W = shape
     rng = np.random.default_rng(Ci + W)
     L = synth.small_random_layer(rng, Co, Ci, P=8, keep=1.0)
@@ -283,9 +283,8 @@ def test_tensor_core_repeatable_multi_tile(pp, runner, oracle_mod, shape, kernel
         for k in range(1, 5):
             assert torch.equal(outs[0], outs[k]), f"run {k} differs from run 0"
         assert pp.pp_layer_device_status(dl.handle) == 0
-        pts = sample_points(rng, N, Co, H, W, 2000)
-        yr, s = oracle_layer_points(oracle_mod, L, x, pts)
-        check_within(outs[0].cpu().numpy()[tuple(pts.T)], yr, s, f"multi-tile {shape}")
+        yr, s = oracle_layer_full(oracle_mod, L, x)
+        check_within(outs[0].cpu().numpy(), yr, s, f"multi-tile {shape}")
     finally:
         dl.close()
 
@@ -436,6 +435,37 @@ def test_single_pattern_layer(pp, runner, oracle_mod, kernel):
     check_within(g, y, s, f"single-pattern layer, {kernel}")
 
 
+@pytest.mark.parametrize("kernel", ["AUTO", "TC", "TC_FLAT", "TMEM", "DIRECT"])
+def test_batchnorm_folded_layer(pp, runner, oracle_mod, kernel):
+    """Section 3's conv + BN fusion: an inference batch normalisation folded into a pruned layer's
+    weights and bias on the host (pp_fold_batchnorm), then packed and run through pp_conv_forward,
+    equals BN applied to the oracle's fp64 conv of the unfolded layer within 1e-5 * S, S the budget of
+    the folded layer (the one-rounding-per-weight fold error is far below it)."""
+    rng = np.random.default_rng(77)
+    Co, Ci, N, H, W = (130, 24, 2, 18, 20) if kernel != "DIRECT" else (12, 3, 2, 18, 20)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.5)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    gamma = rng.uniform(0.5, 2.0, Co).astype(np.float32)
+    beta = rng.normal(0, 0.3, Co).astype(np.float32)
+    mean = rng.normal(0, 0.2, Co).astype(np.float32)
+    var = rng.uniform(0.2, 3.0, Co).astype(np.float32)
+    eps = 1e-5
+    wf, bf = pp.pp_fold_batchnorm(L.w, L.bias, gamma, beta, mean, var, eps)
+    folded = synth.PrunedLayer(w=wf, mask=L.mask, taps=L.taps, bias=bf, pattern_ids=L.pattern_ids)
+    g = run_layer(pp, runner, folded, x, None, True, False,
+                  kernel=None if kernel == "AUTO" else getattr(pp, "PP_KERNEL_" + kernel))
+    # BN(conv(x) + b) in fp64 from the unfolded layer, then ReLU
+    pat = oracle_mod.pattern_ids(L.w, L.mask, L.taps)
+    z, _ = oracle_mod.conv_pruned(x, L.w, pat, L.taps, L.bias)
+    scale = gamma.astype(np.float64) / np.sqrt(var.astype(np.float64) + eps)
+    ybn = (z - mean.astype(np.float64)[None, :, None, None]) * scale[None, :, None, None] + beta.astype(np.float64)[None, :, None, None]
+    ybn = oracle_mod.relu(ybn)
+    # budget of the layer as run: |b'| + sum |w' x|
+    pat_f = oracle_mod.pattern_ids(wf, L.mask, L.taps)
+    _, s = oracle_mod.conv_pruned(x, wf, pat_f, L.taps, bf)
+    check_within(g, ybn, s, f"BN-folded layer, kernel {kernel}")
+
+
 def test_all_pruned_layer_gives_bias(pp, runner, oracle_mod):
     rng = np.random.default_rng(8)
     L = synth.small_random_layer(rng, 20, 10, P=8, keep=0.0)
@@ -465,25 +495,24 @@ def test_cfg0_full(pp, runner, oracle_mod):
     check_within(g, y, s, "cfg0")
 
 
-def layerwise_check(pp, runner, oracle_mod, net, npts, seed=0, check_net=True):
-    """Run a network op by op on the GPU and check every op on sampled outputs against the oracle
-    evaluated on the GPU's own input to that op; then check the executor reproduces the op-by-op
+def layerwise_check(pp, runner, oracle_mod, net, check_net=True, fold_perm=False):
+    """Run a network op by op on the GPU and check every output of every op against the oracle
+    evaluated on the GPU's own input to that op (rearranged into the original channel order when the
+    filter reorder is folded into the next layer); then check the executor reproduces the op-by-op
     result bit for bit (direct launches and CUDA-graph replay) and the host-buffer path too."""
-    rng = np.random.default_rng(seed)
-    dn = runner.DeviceNet(net, use_graph=True)
+    dn = runner.DeviceNet(net, use_graph=True, fold_perm=fold_perm)
     try:
         x = dev(net.x)
         acts = dn.run_layerwise(x)
         torch.cuda.synchronize()
         worst = 0.0
         for k, op in enumerate(net.ops):
-            xin = acts[k].cpu().numpy()
-            out = acts[k + 1].cpu().numpy()
-            skip = acts[op.skip_from].cpu().numpy() if op.skip_from >= 0 else None
-            N, Co, Ho, Wo = out.shape
-            pts = sample_points(rng, N, Co, Ho, Wo, npts)
-            y, s = oracle_layer_points(oracle_mod, op.layer, xin, pts, skip, op.relu, op.pool)
-            worst = max(worst, check_within(out[tuple(pts.T)], y, s, f"{net.name} op {k}"))
+            xin = to_original(acts[k].cpu().numpy(), dn.layouts[k])
+            out = to_original(acts[k + 1].cpu().numpy(), dn.layouts[k + 1])
+            skip = to_original(acts[op.skip_from].cpu().numpy(), dn.layouts[op.skip_from]) if op.skip_from >= 0 else None
+            y, s = oracle_layer_full(oracle_mod, op.layer, xin, skip, op.relu, op.pool)
+            worst = max(worst, check_within(out, y, s, f"{net.name} op {k}"))
+            del y, s, xin, out, skip
         if check_net:
             final = acts[-1]
             y1 = torch.empty_like(final)
@@ -495,22 +524,55 @@ def layerwise_check(pp, runner, oracle_mod, net, npts, seed=0, check_net=True):
             yh = torch.empty(final.shape, dtype=torch.float32).pin_memory()
             dn.run_host(xh, yh)
             assert torch.equal(yh, final.cpu())
+        for L in dn.layers:
+            if not L.dense:
+                assert pp.pp_layer_device_status(L.handle) == 0
         return worst
     finally:
         dn.close()
 
 
 def test_cfg1_vgg16(pp, runner, oracle_mod):
-    assert layerwise_check(pp, runner, oracle_mod, synth.cfg1_vgg16(), 1500) < 1e-5
+    assert layerwise_check(pp, runner, oracle_mod, synth.cfg1_vgg16()) < 1e-5
 
 
 def test_cfg2_style(pp, runner, oracle_mod):
-    assert layerwise_check(pp, runner, oracle_mod, synth.cfg2_style(), 1500) < 1e-5
+    assert layerwise_check(pp, runner, oracle_mod, synth.cfg2_style()) < 1e-5
 
 
-@pytest.mark.slow
 def test_cfg3_vdsr(pp, runner, oracle_mod):
-    assert layerwise_check(pp, runner, oracle_mod, synth.cfg3_vdsr(), 1000) < 1e-5
+    assert layerwise_check(pp, runner, oracle_mod, synth.cfg3_vdsr()) < 1e-5
+
+
+@pytest.mark.parametrize("name", ["vgg16", "style"])
+def test_permutation_folded_networks(pp, runner, oracle_mod, name):
+    """Section 3's filter reorder folded into the next layer (activations kept in reordered channel
+    order between layers, the next layer's input channels permuted at pack time): every op still
+    matches the oracle on every output, the network output is in the original order, and the folded
+    executor reproduces its own op-by-op result bit for bit."""
+    net = synth.cfg1_vgg16() if name == "vgg16" else synth.cfg2_style()
+    assert layerwise_check(pp, runner, oracle_mod, net, fold_perm=True) < 1e-5
+
+
+def test_permutation_folded_layouts(pp, runner):
+    """Which activations the folding keeps in the original order: the network input and output, the
+    skip chain of the style trunk; every other VGG activation is in its producer's reordered order."""
+    dn = runner.DeviceNet(synth.cfg1_vgg16(), use_graph=False, fold_perm=True)
+    try:
+        ident = [bool((l == np.arange(len(l))).all()) for l in dn.layouts]
+        assert ident[0] and ident[-1] and not any(ident[1:-1])
+        for k, L in enumerate(dn.layers[:-1]):
+            assert (dn.layouts[k + 1] == L.perm()).all()
+    finally:
+        dn.close()
+    net = synth.cfg2_style()
+    dn = runner.DeviceNet(net, use_graph=False, fold_perm=True)
+    try:
+        for k, op in enumerate(net.ops):
+            l = dn.layouts[k + 1]
+            assert bool((l == np.arange(len(l))).all()) == (op.skip_from >= 0)
+    finally:
+        dn.close()
 
 
 def test_cfg3_small_full(pp, runner, oracle_mod):
@@ -530,14 +592,23 @@ def test_cfg3_small_full(pp, runner, oracle_mod):
 
 @pytest.mark.parametrize("point", synth.cfg4_points())
 def test_cfg4_sweep_point(pp, runner, oracle_mod, point):
+    """Every output of every sweep point, at the kernel autotuning picks for its shape (as the bench runs it)."""
     C, P, keep = point
     net = synth.cfg4_point(C, P, keep)
     L = net.ops[0].layer
-    g = run_layer(pp, runner, L, net.x)
-    rng = np.random.default_rng(C + P + int(keep * 100))
-    pts = sample_points(rng, *g.shape, 400)
-    y, s = oracle_layer_points(oracle_mod, L, net.x, pts)
-    check_within(g[tuple(pts.T)], y, s, f"sweep {point}")
+    N, _, H, W = net.x.shape
+    dl = runner.DeviceLayer(L)
+    try:
+        pp.pp_layer_autotune(dl.handle, N, H, W, 0, torch.cuda.current_stream())
+        y = torch.full((N, C, H, W), float("nan"), device="cuda")
+        dl.forward(dev(net.x), y, None, N, H, W, 0, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        assert pp.pp_layer_device_status(dl.handle) == 0
+        g = y.cpu().numpy()
+    finally:
+        dl.close()
+    yr, s = oracle_layer_full(oracle_mod, L, net.x)
+    check_within(g, yr, s, f"sweep {point}")
 
 
 def test_bad_arguments_rejected(pp, runner):
@@ -619,3 +690,53 @@ def run_host_paths(pp, runner, spec):
             assert torch.equal(o, ref)
     finally:
         dn.close()
+
+
+@pytest.mark.parametrize("kernel", ["TC", "TC_FLAT", "TMEM", "REGISTER", "DIRECT"])
+def test_output_order_every_kernel(pp, runner, oracle_mod, kernel):
+    """pp_layer_set_output_order: original filter o lands in channel order[o] on every kernel (skip read at
+    the same channel, pooling included), NULL restores the original order."""
+    rng = np.random.default_rng(91)
+    Co, Ci = (12, 3) if kernel == "DIRECT" else (136, 24)
+    N, H, W = 2, 14, 18
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.5)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32)
+    order = rng.permutation(Co).astype(np.int32)
+    flags = pp.PP_ADD_SKIP | pp.PP_RELU | pp.PP_POOL2
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, True, True)
+    dl = runner.DeviceLayer(L)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, getattr(pp, "PP_KERNEL_" + kernel))
+        for ordv in (order, None):
+            pp.pp_layer_set_output_order(dl.handle, ordv, torch.cuda.current_stream())
+            sk = skip.copy()
+            if ordv is not None:
+                sk[:, ordv] = skip  # the skip tensor in the output's channel order
+            out = torch.full((N, Co, H // 2, W // 2), float("nan"), device="cuda")
+            dl.forward(dev(x), out, dev(sk), N, H, W, flags, torch.cuda.current_stream())
+            torch.cuda.synchronize()
+            g = out.cpu().numpy()
+            g = g[:, ordv] if ordv is not None else g  # back to the original order
+            check_within(g, y, s, f"output order {kernel} {'set' if ordv is not None else 'reset'}")
+        bad = order.copy()
+        bad[0] = bad[1]
+        with pytest.raises(pp.PPError) as e:
+            pp.pp_layer_set_output_order(dl.handle, bad, torch.cuda.current_stream())
+        assert e.value.code == pp.PP_ERR_INVALID_ARG
+    finally:
+        dl.close()
+
+
+def test_peak_probes(pp):
+    """pp_peak_probe: the FFMA probe runs near the FP32 lanes' rate at the SM clock it reports, and the
+    tensor-core probes well above it (f16 above tf32)."""
+    props = torch.cuda.get_device_properties(0)
+    tf, mhz, ms = pp.pp_peak_probe(pp.PP_PROBE_FFMA, 1 << 14)
+    assert 300 < mhz < 2500 and ms > 0
+    lanes_rate = props.multi_processor_count * 128 * 2 * mhz * 1e6 / 1e12
+    assert 0.5 * lanes_rate < tf < 1.05 * lanes_rate, (tf, lanes_rate)
+    t32, m32, _ = pp.pp_peak_probe(pp.PP_PROBE_MMA_TF32, 1 << 12)
+    t16, m16, _ = pp.pp_peak_probe(pp.PP_PROBE_MMA_F16, 1 << 12)
+    assert t32 > 5 * tf and t16 > 1.3 * t32, (tf, t32, t16)
+    assert 300 < m32 < 2500 and 300 < m16 < 2500

@@ -1,13 +1,19 @@
-"""pp_conv_forward_noalloc: the flat tensor-core kernel with its split partials in
-a static device array, against pp_conv_forward on the same layer.  Kept in its
-own file, named to be collected last, so it runs both alone in a fresh process
-and after every other GPU test."""
+"""pp_conv_forward_noalloc: the flat tensor-core kernel run without any device
+allocation by the call, for callers that cannot allocate while they run layers
+(their device memory is reserved up front by another allocator, or their loop
+cannot take the device-wide synchronisation of cudaMalloc / cudaFree).  Its
+cluster-split partial tiles are reduced through distributed shared memory, so
+the call needs no workspace.  Checked against pp_conv_forward and the oracle on
+two calls in a row, with an unsplit (persistent) and a split geometry pinned,
+on a layer whose selected kernel is another one, and against the device's free
+memory.  Kept in its own file, named to be collected last, so it runs both
+alone in a fresh process and after every other GPU test."""
 import numpy as np
 import pytest
 import torch
 
 from paper_2004_11250_gb300 import synth
-from parity import check_within, oracle_layer_points, sample_points
+from parity import check_within, oracle_layer_full
 
 pytestmark = pytest.mark.gpu
 
@@ -21,9 +27,17 @@ def pp():
     return ppconv
 
 
-@pytest.mark.parametrize("shape,flags", [((1, 512, 512, 14, 14), "relu"), ((1, 256, 512, 28, 28), "pool_relu"),
-                                         ((2, 64, 200, 20, 30), "skip_relu")])
-def test_noalloc_matches_forward(pp, oracle_mod, shape, flags):
+# (N, Ci, Co, H, W), flags, pinned (R, S) or None, kernel the layer keeps selected
+CASES = [
+    ((1, 512, 512, 14, 14), "relu", (14, 4), "TC_FLAT"),      # cluster split, read back through the pin
+    ((4, 128, 256, 28, 28), "pool_relu", (8, 1), "TC_FLAT"),  # unsplit, persistent over tiles
+    ((2, 64, 200, 20, 30), "skip_relu", None, "TC"),          # the layer runs the row-tiled kernel otherwise
+    ((1, 96, 144, 16, 24), "relu", None, "REGISTER"),         # ... or an FMA kernel
+]
+
+
+@pytest.mark.parametrize("shape,flags,geo,kernel", CASES)
+def test_noalloc_matches_forward(pp, oracle_mod, shape, flags, geo, kernel):
     from paper_2004_11250_gb300 import runner
     N, Ci, Co, H, W = shape
     rng = np.random.default_rng(Ci + Co + W)
@@ -35,29 +49,36 @@ def test_noalloc_matches_forward(pp, oracle_mod, shape, flags):
     Ho, Wo = (H // 2, W // 2) if pool else (H, W)
     dl = runner.DeviceLayer(L)
     try:
-        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC_FLAT)
+        pp.pp_layer_set_kernel(dl.handle, getattr(pp, "PP_KERNEL_" + kernel))
+        if geo is not None:
+            pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, f, *geo)
+            assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, f) == geo
         xd = torch.from_numpy(x).cuda()
         sd = None if skip is None else torch.from_numpy(skip).cuda()
         ref = torch.full((N, Co, Ho, Wo), float("nan"), device="cuda")
         dl.forward(xd, ref, sd, N, H, W, f, torch.cuda.current_stream())
-        outs = []
-        for _ in range(2):  # two calls in a row reuse the static workspace
-            y = torch.full((N, Co, Ho, Wo), float("nan"), device="cuda")
-            pp.pp_conv_forward_noalloc(dl.handle, xd, y, sd, N, H, W, f, torch.cuda.current_stream())
-            outs.append(y)
+        outs = [torch.full((N, Co, Ho, Wo), float("nan"), device="cuda") for _ in range(3)]
+        # a first call loads the kernel's code (lazy module loading) and sets its attributes
+        pp.pp_conv_forward_noalloc(dl.handle, xd, outs.pop(), sd, N, H, W, f, torch.cuda.current_stream())
         torch.cuda.synchronize()
+        free0, _ = torch.cuda.mem_get_info()
+        for y in outs:  # two calls in a row on the same layer
+            pp.pp_conv_forward_noalloc(dl.handle, xd, y, sd, N, H, W, f, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        free1, _ = torch.cuda.mem_get_info()
+        assert free1 == free0, "the call changed the device's free memory"
         assert pp.pp_layer_device_status(dl.handle) == 0
-        pts = sample_points(rng, N, Co, Ho, Wo, 1500)
-        yr, s = oracle_layer_points(oracle_mod, L, x, pts, skip, True, pool)
-        idx = tuple(pts.T)
+        assert pp.pp_layer_kernel(dl.handle) == getattr(pp, "PP_KERNEL_" + kernel)  # selection untouched
+        yr, s = oracle_layer_full(oracle_mod, L, x, skip, True, pool)
         r = ref.cpu().numpy()
         for k, y in enumerate(outs):
             g = y.cpu().numpy()
             assert np.isfinite(g).all(), f"call {k}: outputs left unwritten"
             # the two entry points agree within the tests' bound of each other ...
-            check_within(g[idx], r[idx].astype(np.float64), s, f"noalloc call {k} vs pp_conv_forward")
+            check_within(g, r.astype(np.float64), s, f"noalloc call {k} vs pp_conv_forward")
             # ... and with the oracle
-            check_within(g[idx], yr, s, f"noalloc call {k} vs oracle")
+            check_within(g, yr, s, f"noalloc call {k} vs oracle")
+        assert torch.equal(outs[0], outs[1])
     finally:
         dl.close()
 
