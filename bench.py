@@ -343,30 +343,31 @@ def kernel_source_hash():
 TENSOR_PEAKS = {}  # filled by main(): {"tf32": TFLOP/s, "f16": TFLOP/s} measured by pp_peak_probe
 
 
-def tensor_view(shapes, kern, op_ms, pruned):
+def tensor_view(shapes, kern, op_ms, pruned, f16=False):
     """Tensor-pipe view of the pruned ops that run on a tensor-core kernel: their dense 9-tap contraction
-    in 3 tf32 passes (hi*hi, lo*hi, hi*lo) per second against the measured kind::tf32 MMA peak; None
-    without such ops."""
+    in 3 passes (hi*hi, lo*hi, hi*lo) per second against the measured kind::tf32 (or kind::f16) MMA
+    peak; None without such ops."""
     tc_ops = [k for k in pruned if kern[k] in ("ppconv_tc_kernel", "ppconv_tcf_kernel")]
-    if not tc_ops or "tf32" not in TENSOR_PEAKS:
+    kind = "f16" if f16 else "tf32"
+    if not tc_ops or kind not in TENSOR_PEAKS:
         return None
     tf = sum(3 * 2 * shapes[k]["N"] * shapes[k]["Ci"] * shapes[k]["Co"] * 9 * shapes[k]["H"] * shapes[k]["W"]
              for k in tc_ops)
     tt = sum(op_ms[k] for k in tc_ops) * 1e-3
-    tpk = TENSOR_PEAKS["tf32"]
+    tpk = TENSOR_PEAKS[kind]
     return {"bound": "tensor", "ops": len(tc_ops), "achieved": round(tf / tt / 1e12, 2), "peak": round(tpk, 1),
-            "unit": "TFLOP/s (tf32, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
-            "peak_source": "measured: pp_peak_probe kind::tf32 MMA (M 128, N 256, K 8), this run"}
+            "unit": f"TFLOP/s ({kind}, dense 9-tap, 3 passes)", "frac": round(tf / tt / 1e12 / tpk, 4),
+            "peak_source": f"measured: pp_peak_probe kind::{kind} MMA (M 128, N 256, K {16 if f16 else 8}), this run"}
 
 
-def bench_config(name, steps, warmup, flush, stream, hbm, fold_too=False):
+def bench_config(name, steps, warmup, flush, stream, hbm, fold_too=False, precision=0):
     """ms/frame, GFLOP/s and per-op roofline fractions (op times taken inside the frame) of one workload,
     for the all-configs table; with fold_too also the frame time with the filter reorder folded into the
     next layer (Section 3 matrix reorder; activations between layers in reordered channel order)."""
     import torch
     from paper_2004_11250_gb300 import runner
     spec = workload(name)
-    dn = runner.DeviceNet(spec, use_graph=True)
+    dn = runner.DeviceNet(spec, use_graph=True, precision=precision)
     try:
         x = torch.from_numpy(spec.x).cuda()
         y = torch.empty(dn.out_shape, device="cuda")
@@ -382,7 +383,7 @@ def bench_config(name, steps, warmup, flush, stream, hbm, fold_too=False):
         from paper_2004_11250_gb300 import ppconv as pp
         per_op = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "dense" for L in dn.layers]
         kern = sorted(set(k for k in per_op if k != "dense"))
-        tv = tensor_view(shapes, per_op, op_ms, [k for k, s in enumerate(shapes) if s["pruned"]])
+        tv = tensor_view(shapes, per_op, op_ms, [k for k, s in enumerate(shapes) if s["pruned"]], f16=precision == 1)
         res = {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1), "kernels": kern,
                "op_us_in_frame": [round(t * 1e3, 2) for t in op_ms],
                "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
@@ -402,7 +403,7 @@ def bench_config(name, steps, warmup, flush, stream, hbm, fold_too=False):
     return res
 
 
-def bench_sweep(steps, flush, stream, hbm):
+def bench_sweep(steps, flush, stream, hbm, precision=0):
     """Sweep workload: per point (C, P, keep) one layer at 8x56x56, its kernel autotuned at that shape;
     returns summary + per-point roofline fractions and the kernel used."""
     import torch
@@ -410,7 +411,7 @@ def bench_sweep(steps, flush, stream, hbm):
     fracs, total_ms = {}, 0.0
     for (C, P, keep) in synth.cfg4_points():
         spec = synth.cfg4_point(C, P, keep)
-        L = runner.DeviceLayer(spec.ops[0].layer)
+        L = runner.DeviceLayer(spec.ops[0].layer, precision=precision)
         try:
             from paper_2004_11250_gb300 import ppconv as pp
             pp.pp_layer_autotune(L.handle, 8, 56, 56, 0, stream)  # kernel choice at this shape, before timing
@@ -531,6 +532,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="vgg16",
                     help="vgg16 (default), single, style, vdsr, or sweep:C:P:keep (one point of the sweep)")
+    ap.add_argument("--precision", default="tf32x3", choices=["tf32x3", "f16x3"],
+                    help="arithmetic of the tensor-core kernels for the timed frames (pp_layer_set_precision)")
     ap.add_argument("--fold-perm", action="store_true",
                     help="fold each layer's filter reorder into the next layer for the timed frames")
     ap.add_argument("--no-configs", action="store_true", help="skip the all-configs table")
@@ -564,7 +567,8 @@ def main():
     spec = workload(args.workload)
     shapes = op_shapes(spec)
     flops_frame = sum(s["flops"] for s in shapes)
-    dn = runner.DeviceNet(spec, use_graph=True, fold_perm=args.fold_perm)
+    precision = 1 if args.precision == "f16x3" else 0
+    dn = runner.DeviceNet(spec, use_graph=True, fold_perm=args.fold_perm, precision=precision)
     if args.kernels:
         from paper_2004_11250_gb300 import ppconv as pp
         ids = {"tm": pp.PP_KERNEL_TMEM, "reg": pp.PP_KERNEL_REGISTER, "tc": pp.PP_KERNEL_TC,
@@ -621,7 +625,7 @@ def main():
             R, S = pp.pp_layer_flat_geometry(L.handle, sh["N"], sh["H"], sh["W"], runner.op_flags(op))
             g = f"{R}:{S}" if R else "model"
         geo.append(g)
-    tensor = tensor_view(shapes, kern, op_ms, pruned)
+    tensor = tensor_view(shapes, kern, op_ms, pruned, f16=precision == 1)
     # the dominant kernel (most device time over the pruned ops): its surviving FLOPs per launch over
     # its mean launch duration, against the FP32 roofline of the method
     by_kern = {}
@@ -654,7 +658,10 @@ def main():
         configs = {}
         for name in ("single", "vgg16", "style", "vdsr"):
             configs[name] = bench_config(name, 10, 3, flush, stream, hbm, fold_too=name in ("vgg16", "style"))
+            if name != "single":  # the single 16-channel layer has no tensor-core layout
+                configs[name]["f16x3"] = bench_config(name, 10, 3, flush, stream, hbm, precision=1)
         configs["sweep"] = bench_sweep(5, flush, stream, hbm)
+        configs["sweep"]["f16x3"] = bench_sweep(5, flush, stream, hbm, precision=1)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
@@ -684,7 +691,8 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded; shapes and distributions of the workload, no dataset or trained weights)",
-            "config": dict(config_dict(args.workload), perm_folded=bool(args.fold_perm)),
+            "config": dict(config_dict(args.workload), perm_folded=bool(args.fold_perm),
+                           tensor_core_precision=args.precision),
             "e2e": {"value": round(e2e_value, 2), "unit": "GFLOP/s", "h2d_bytes_per_step": int(xh.numel() * 4),
                     "d2h_bytes_per_step": int(yh.numel() * 4), "ms_per_step": round(statistics.median(e2e_t) * 1e3, 4)},
             "gpu_launches": len(spec.ops) * args.steps,

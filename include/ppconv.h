@@ -207,6 +207,41 @@ pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* 
  * Errors: PP_ERR_INVALID_ARG (not a permutation), PP_ERR_CUDA, PP_ERR_OOM. */
 pp_status pp_layer_set_output_order(pp_layer* layer, const int32_t* order, void* stream);
 
+/*
+ * Arithmetic of the tensor-core kernels (PP_KERNEL_TC, PP_KERNEL_TC_FLAT and
+ * pp_conv_forward_noalloc); the FMA kernels always compute in fp32.  Both
+ * modes meet |gpu - exact| <= 1e-5 * S (S = |bias| + sum |w x| + |skip|) on
+ * the inputs their conditions cover.
+ *   PP_PRECISION_TF32X3  the default: each operand v = hi + lo with hi its
+ *       tf32 truncation; w_hi x_hi + w_lo x_hi + w_hi x_lo accumulated in fp32
+ *       (tcgen05 kind::tf32).  Any fp32 input.
+ *   PP_PRECISION_F16X3   each operand v = hi + 2^-11 lo with hi = f16(v) and
+ *       lo = f16((v - hi) 2^11), rounded to nearest, after exact power-of-two
+ *       scaling: per filter for the weights (largest kept |w| into
+ *       [2^13, 2^14)), per layer for the input (x_s = x * s_x, s_x the largest
+ *       power of two with input_bound * s_x <= 2^14); w_hi x_hi into one fp32
+ *       accumulator, w_lo x_hi + w_hi x_lo into a second (tcgen05 kind::f16,
+ *       twice the tf32 rate on half the operand bytes), combined as
+ *       (acc1 + 2^-11 acc2) / (s_w s_x).  Per product the representation
+ *       error is below 3 * 2^-22 of |w x| while |x_s| >= 2^-14; below that
+ *       fp16's subnormal spacing adds at most 2^-36 / s_x per unit of |w|, so
+ *       the bound holds unless an output's whole receptive field is tiny
+ *       (mean |x| below ~1e-6 / s_x) yet not zero.  Inputs must satisfy
+ *       |x_s| < 2^15 (|x| < 2 * input_bound at least); a launch that meets a
+ *       larger one sets bit 1 of the layer's device status word and its
+ *       output is invalid.  input_bound <= 0 means 16384 (s_x = 1).
+ * Switching to PP_PRECISION_F16X3 builds the f16 weight layout (half the
+ * bytes of the tf32 one) from a host copy of the packed layer, synchronously
+ * on stream; a CUDA graph captured before keeps the old arithmetic.
+ * Errors: PP_ERR_INVALID_ARG (unknown precision, NaN bound), PP_ERR_UNSUPPORTED
+ * (F16X3 on a layer without a tensor-core layout: Ci < 8), PP_ERR_CUDA,
+ * PP_ERR_OOM. */
+#define PP_PRECISION_TF32X3 0
+#define PP_PRECISION_F16X3 1
+pp_status pp_layer_set_precision(pp_layer* layer, int precision, float input_bound, void* stream);
+/* The layer's precision and input scale s_x (1 under PP_PRECISION_TF32X3); either pointer may be NULL. */
+pp_status pp_layer_precision(const pp_layer* layer, int* precision, float* input_scale);
+
 /* Which kernel pp_conv_forward runs for a layer.  All compute the same
  * convolution within the documented fp32 bound.
  *   PP_KERNEL_TC        implicit GEMM on the tensor cores over the 9 taps
@@ -270,8 +305,11 @@ pp_status pp_layer_autotune(pp_layer* layer, int N, int H, int W, int flags, voi
 pp_status pp_layer_flat_geometry(const pp_layer* layer, int N, int H, int W, int flags, int* R, int* S);
 pp_status pp_layer_pin_flat_geometry(pp_layer* layer, int N, int H, int W, int flags, int R, int S);
 
-/* Synchronous: *device_error = 0 unless a kernel of this layer gave up a
- * bounded wait (its output is then invalid); the word is cleared by the read. */
+/* Synchronous: *device_error = 0 unless a launch of this layer's tensor-core
+ * kernels met an error since the last read, and its output is then invalid:
+ * bit 0 (value 1) a bounded wait gave up; bit 1 (value 2) under
+ * PP_PRECISION_F16X3 an input was at or beyond 2^15 after the layer's input
+ * scale.  The word is cleared by the read. */
 pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);
 
 /* Polls of an mbarrier after which a wait in the tensor-core kernels gives up:

@@ -38,6 +38,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -415,6 +416,8 @@ struct pp_layer {
   std::vector<int32_t> pk_perm;     // the packer's filter permutation (host copy)
   std::vector<float> direct_w;      // direct layout's dense weights [Co][Ci][9], original filter order
   std::vector<float> direct_bias;   // and its bias (empty: none)
+  pp_packed packed;                 // host copy of the packed layer (tensor-core layers: f16 layout built on demand)
+  int precision = PP_PRECISION_TF32X3;
 };
 
 struct pp_dense {
@@ -687,6 +690,7 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
     st = ppc::tc_prepare();
     if (st == PP_OK) st = ppc::tc_build(&L->tc, pk, (cudaStream_t)stream);
     L->tc_ok = st == PP_OK;
+    if (L->tc_ok) L->packed = *pk;
   }
   if (st == PP_OK && ppc::direct_applicable(pk->Co, pk->Ci)) {
     // dense [Co][Ci][9] in the original filter order, zeros where pruned
@@ -755,6 +759,29 @@ extern "C" pp_status pp_layer_set_output_order(pp_layer* L, const int32_t* order
     ppc::direct_free(&L->direct);
     L->direct = D;
   }
+  return PP_OK;
+}
+
+extern "C" pp_status pp_layer_set_precision(pp_layer* L, int precision, float input_bound, void* stream) {
+  if (!L) return PP_ERR_INVALID_ARG;
+  if (precision == PP_PRECISION_TF32X3) {
+    L->tc.f16 = false;
+    L->precision = precision;
+    return PP_OK;
+  }
+  if (precision != PP_PRECISION_F16X3 || std::isnan(input_bound)) return PP_ERR_INVALID_ARG;
+  if (!L->tc_ok) return PP_ERR_UNSUPPORTED;
+  const pp_status st = ppc::tc_build16(&L->tc, &L->packed, input_bound, (cudaStream_t)stream);
+  if (st != PP_OK) return st;
+  L->tc.f16 = true;
+  L->precision = precision;
+  return PP_OK;
+}
+
+extern "C" pp_status pp_layer_precision(const pp_layer* L, int* precision, float* input_scale) {
+  if (!L) return PP_ERR_INVALID_ARG;
+  if (precision) *precision = L->precision;
+  if (input_scale) *input_scale = L->precision == PP_PRECISION_F16X3 ? L->tc.xscale : 1.f;
   return PP_OK;
 }
 
@@ -897,7 +924,7 @@ extern "C" pp_status pp_layer_info(const pp_layer* L, int* Co, int* Ci, int64_t*
   if (Co) *Co = L->Co;
   if (Ci) *Ci = L->Ci;
   if (device_bytes)
-    *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes + L->tc.dbytes +
+    *device_bytes = (int64_t)(L->dbytes + L->tm.dbytes + L->tc.dbytes + L->tc.dbytes16 +
                               (L->direct.w ? ((size_t)L->Co * L->Ci * 9 + (L->direct.bias ? L->Co : 0)) * 4 : 0));
   return PP_OK;
 }

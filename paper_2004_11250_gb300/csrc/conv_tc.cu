@@ -35,6 +35,14 @@
 //     2 (x_hi [w_hi | w_lo] as one 2 FB-wide operand, then x_lo w_hi);
 //   * tcgen05.commit signals an mbarrier when the chunk's MMAs have read their
 //     operands, which frees that stage for the chunk after next.
+// fp16 split (layers set to PP_PRECISION_F16X3, F16 instantiations): operands
+// held as hi = f16(v) and lo = f16((v - hi) * 2^11) (weights scaled per filter,
+// the input per layer, by powers of two), 16-channel chunks (the K of
+// kind::f16), w_hi x_hi into one accumulator and w_lo x_hi + w_hi x_lo into a
+// second one (pixel-major: the lo half of the merged operand's columns and the
+// x_lo MMA; filter-major: the row segment's second TW columns), combined in the
+// epilogue as (acc1 + 2^-11 acc2) times the filter's inverse scale; inputs at
+// or beyond 2^15 after scaling are flagged in the device status word.
 // Epilogue: bias, +skip, ReLU, 2x2 max pool from tcgen05.ld, stores to each
 // filter's original channel.  This kernel has no channel split: layers with
 // more than 64 filters on maps at most 128 wide can also run the flat kernel
@@ -46,7 +54,10 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <cuda_fp16.h>
+
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -78,6 +89,8 @@ constexpr long WAIT_LIMIT = PP_WAIT_POLLS;  // mbarrier polls before a wait give
 enum { ORI_FP = 0, ORI_PF = 1, ORI_PFR = 2 };
 
 struct TcParams {
+  const float* rscale;      // f16: per reordered filter, 1 / (weight scale x input scale)
+  float xscale;             // f16: power of two applied to x before the split
   const float* x;
   float* y;
   const float* skip;
@@ -94,17 +107,21 @@ struct TcParams {
 
 // Geometry of one instantiation.  TW pixels per output row segment, FB filters
 // per block, R row segments per tile (one accumulator column range each).
-template <int ORI, int TW, int FB>
+template <int ORI, int TW, int FB, bool F16>
 struct Geo {
   static_assert(ORI == ORI_FP ? FB == 128 : (ORI == ORI_PF ? TW == 128 : (128 % TW == 0 && FB == 64)),
                 "orientation needs a 128-row M side");
+  static constexpr int KCH = F16 ? 16 : KC;  // input channels per chunk
+  static constexpr int CPH = KCH / 2;        // channels per K half (16 bytes of a pixel's operand row)
   // MRG (pixel-major): the hi and lo weight tiles of a tap are one 2 FB-wide B
   // operand, so x_hi * [w_hi | w_lo] is one N = 2 FB MMA (the lo part lands in
   // accumulator columns FB .. 2 FB - 1 and the epilogue adds the two halves);
   // x_lo * w_hi is an N = FB MMA.  Two MMAs instead of three read the pixel
   // tile twice instead of three times.
   static constexpr bool MRG = ORI != ORI_FP;
-  static constexpr int SEGC = ORI == ORI_FP ? TW : (MRG ? 2 * FB : FB);  // accumulator columns per row segment
+  // accumulator columns per row segment (f16 filter-major: a second accumulator of TW columns follows)
+  static constexpr int SEGC = ORI == ORI_FP ? (F16 ? 2 * TW : TW) : (MRG ? 2 * FB : FB);
+  static constexpr int ACC2 = ORI == ORI_FP ? TW : FB;   // f16: offset of the second accumulator in a segment
   static constexpr int NSEG = NCOL / SEGC;                // MMA row segments per tile
   static constexpr int RSEG = ORI == ORI_PFR ? 128 / TW : 1;  // output rows per segment
   static constexpr int R = NSEG * RSEG;                   // output rows per tile
@@ -118,9 +135,9 @@ struct Geo {
   // tensor-map box width: columns c0-4 .. (staged column bc is box column bc + 3),
   // a multiple of 4 so each box row is whole 16-byte units
   static constexpr int RAW_W = (BCOLS + 3 + 3) / 4 * 4;
-  static constexpr int RAW = KC * BROWS * RAW_W * 4;      // box [8 channels][BROWS][RAW_W], landed in the lo area
+  static constexpr int RAW = KCH * BROWS * RAW_W * 4;     // box [KCH channels][BROWS][RAW_W], landed in the lo area
   static constexpr int LO_BYTES = IN_BYTES > RAW ? IN_BYTES : RAW;
-  static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo
+  static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo (FB x 8 fp32 or FB x 16 f16)
   static constexpr int W_BYTES = NTAP * 2 * W_TILE;       // weights of one chunk
   // SEP: the raw boxes get a ring of their own (two slots), so the copy for a
   // chunk can start two chunks ahead instead of waiting for the MMAs that read
@@ -132,8 +149,9 @@ struct Geo {
   static constexpr int SMEM_ALLOC = 2 * STAGE + (SEP ? 2 * RAW : 0) + 1024;
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
   static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
-  static constexpr uint32_t IDESC = ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB);
-  static constexpr uint32_t IDESC2 = idesc_tf32(128, 2 * FB);  // MRG: [w_hi | w_lo]
+  static constexpr uint32_t IDESC = F16 ? (ORI == ORI_FP ? idesc_f16(128, TW) : idesc_f16(128, FB))
+                                        : (ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB));
+  static constexpr uint32_t IDESC2 = F16 ? idesc_f16(128, 2 * FB) : idesc_tf32(128, 2 * FB);  // MRG: [w_hi | w_lo]
   static constexpr int WLBO = 2 * FB * 16;  // weights: bytes between K halves (hi and lo rows of a tap in each)
 };
 
@@ -153,9 +171,9 @@ __device__ __forceinline__ Tile tile_of(const TcParams& p, int t, int R, int TW)
   return T;
 }
 
-template <int ORI, int TW, int FB>
+template <int ORI, int TW, int FB, bool F16>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p, const __grid_constant__ CUtensorMap xmap) {
-  using G = Geo<ORI, TW, FB>;
+  using G = Geo<ORI, TW, FB, F16>;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // Offset from the shared array itself (not an integer round trip), so the
   // compiler keeps every access below in the shared state space.
@@ -174,7 +192,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       if ((i & 255) == 255 && abort_s) return false;
     }
     abort_s = 1;
-    atomicExch(p.status, 1);
+    atomicOr(p.status, ppc::kStatusTimeout);
     return false;
   };
 
@@ -217,7 +235,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       asm volatile(
           "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
           "%4, %5}], [%6];" ::"r"(su32(dst)),
-          "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(T.c0 - 4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
+          "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(T.c0 - 4), "r"(T.r0 - 1), "r"(c * G::KCH), "r"(T.n),
           "r"(su32(&raw_full[gg & 1]))
           : "memory");
     };
@@ -243,6 +261,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + G::RAW_OFF + raw_issued * G::RAW);
     int g = 0;  // chunk sequence number of this CTA
     bool stop = false;  // identical in every loader thread (decided by loader_any)
+    bool range_bad = false;  // f16: an input at or beyond 2^15 after scaling
     for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
@@ -265,7 +284,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             ++raw_issued;
           }
         }
-        const int ch0 = c * KC;
+        const int ch0 = c * G::KCH;
         if (p.use_tma) {
           if (group_any<NLOAD>(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
             stop = true;
@@ -273,7 +292,34 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           }
           const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g & 1) * G::RAW)
                                     : reinterpret_cast<const float*>(lo);
-          float v[G::ITEMS][4];
+          if constexpr (F16 && G::SEP) {
+            // the box has a slot of its own: each item is split and stored as soon as it is read (fewer
+            // live registers than reading the whole box first); the slot is released after the last read
+#pragma unroll
+            for (int b = 0; b < G::ITEMS; ++b) {
+              const int it = b * NLOAD + tid;
+              if (it < 2 * G::NPIX) {
+                const int kh = it >= G::NPIX ? 1 : 0;
+                const int pix = it - kh * G::NPIX;
+                const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
+                float u[G::CPH];
+#pragma unroll
+                for (int k = 0; k < G::CPH; ++k) u[k] = raw[((kh * G::CPH + k) * G::BROWS + br) * G::RAW_W + bc + 3];
+                uint4 h, l;
+                range_bad |= split_f16x8(u, p.xscale, h, l);
+                const int dst = it + (kh ? G::NPIXA - G::NPIX : 0);  // K halves NPIXA apart
+                reinterpret_cast<uint4*>(hi)[dst] = h;
+                reinterpret_cast<uint4*>(lo)[dst] = l;
+              }
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            group_sync<NLOAD>();
+            if (tid == 0 && raw_issued < nall && raw_issued == g + 2) {
+              issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued & 1) * G::RAW);
+              ++raw_issued;
+            }
+          } else {
+          float v[G::ITEMS][G::CPH];
 #pragma unroll
           for (int b = 0; b < G::ITEMS; ++b) {
             const int it = b * NLOAD + tid;
@@ -281,8 +327,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             const int pix = it - kh * G::NPIX;
             const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              v[b][k] = it < 2 * G::NPIX ? raw[((kh * 4 + k) * G::BROWS + br) * G::RAW_W + bc + 3] : 0.f;
+            for (int k = 0; k < G::CPH; ++k)
+              v[b][k] = it < 2 * G::NPIX ? raw[((kh * G::CPH + k) * G::BROWS + br) * G::RAW_W + bc + 3] : 0.f;
           }
           // The raw slot is rewritten next by a tensor-map copy (async proxy):
           // each thread orders its generic-proxy reads of the slot before that
@@ -297,21 +343,29 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           for (int b = 0; b < G::ITEMS; ++b) {
             const int it = b * NLOAD + tid;
             if (it < 2 * G::NPIX) {
-              float4 h;
-              h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
-              h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
-              h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
-              h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
               const int dst = it + (it >= G::NPIX ? G::NPIXA - G::NPIX : 0);  // K halves NPIXA apart
-              hi[dst] = h;
-              lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+              if constexpr (F16) {
+                uint4 h, l;
+                range_bad |= split_f16x8(&v[b][0], p.xscale, h, l);
+                reinterpret_cast<uint4*>(hi)[dst] = h;
+                reinterpret_cast<uint4*>(lo)[dst] = l;
+              } else {
+                float4 h;
+                h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
+                h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
+                h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
+                h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
+                hi[dst] = h;
+                lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+              }
             }
+          }
           }
         } else {
           // Items in batches of LBATCH per thread: all global loads of a batch
           // are issued before any is used, so their latencies overlap.
           for (int base = 0; base < 2 * G::NPIX; base += NLOAD * LBATCH) {
-            float v[LBATCH][4];
+            float v[LBATCH][G::CPH];
 #pragma unroll
             for (int b = 0; b < LBATCH; ++b) {
               const int it = base + b * NLOAD + tid;
@@ -321,8 +375,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               const int r = T.r0 - 1 + br, cc = T.c0 - 1 + bc;
               const bool inside = it < 2 * G::NPIX && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
 #pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                const int ch = ch0 + kh * 4 + k;
+              for (int k = 0; k < G::CPH; ++k) {
+                const int ch = ch0 + kh * G::CPH + k;
                 v[b][k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
               }
             }
@@ -330,14 +384,21 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             for (int b = 0; b < LBATCH; ++b) {
               const int it = base + b * NLOAD + tid;
               if (it < 2 * G::NPIX) {
-                float4 h;
-                h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
-                h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
-                h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
-                h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
                 const int dst = it + (it >= G::NPIX ? G::NPIXA - G::NPIX : 0);
-                hi[dst] = h;
-                lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+                if constexpr (F16) {
+                  uint4 h, l;
+                  range_bad |= split_f16x8(&v[b][0], p.xscale, h, l);
+                  reinterpret_cast<uint4*>(hi)[dst] = h;
+                  reinterpret_cast<uint4*>(lo)[dst] = l;
+                } else {
+                  float4 h;
+                  h.x = __uint_as_float(__float_as_uint(v[b][0]) & 0xFFFFE000u);
+                  h.y = __uint_as_float(__float_as_uint(v[b][1]) & 0xFFFFE000u);
+                  h.z = __uint_as_float(__float_as_uint(v[b][2]) & 0xFFFFE000u);
+                  h.w = __uint_as_float(__float_as_uint(v[b][3]) & 0xFFFFE000u);
+                  hi[dst] = h;
+                  lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+                }
               }
             }
           }
@@ -346,6 +407,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         mbar_arrive(su32(&full[s]));
       }
     }
+    if (F16 && range_bad) atomicOr(p.status, ppc::kStatusF16Range);
     if (tid == 0) {
       // No copy may still be writing shared memory when the CTA exits: after an
       // early stop, wait (bounded) for the last copies of each kind to land.
@@ -392,7 +454,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               const uint64_t off = (uint64_t)((rr * G::RSEG + dy) * G::BCOLS + dx);  // pixels of 16 bytes
               const uint64_t xh = xh0 + off, xl = xl0 + off;
               const uint32_t d = dbase + (uint32_t)(rr * G::SEGC);
-              if (ORI == ORI_FP) {
+              if (F16) {
+                // acc1 += w_hi x_hi; acc2 += w_lo x_hi + w_hi x_lo (lo parts scaled by 2^11)
+                if (ORI == ORI_FP) {
+                  mma_f16(d, whi, xh, G::IDESC, t == 0 ? acc0 : 1u);
+                  mma_f16(d + G::ACC2, wlo, xh, G::IDESC, t == 0 ? acc0 : 1u);
+                  mma_f16(d + G::ACC2, whi, xl, G::IDESC, 1u);
+                } else {
+                  mma_f16(d, xh, whi, G::IDESC2, t == 0 ? acc0 : 1u);  // [acc1 | acc2] += x_hi [w_hi | w_lo]
+                  mma_f16(d + G::ACC2, xl, whi, G::IDESC, 1u);
+                }
+              } else if (ORI == ORI_FP) {
                 mma_tf32(d, whi, xh, G::IDESC, t == 0 ? acc0 : 1u);
                 mma_tf32(d, wlo, xh, G::IDESC, 1u);
                 mma_tf32(d, whi, xl, G::IDESC, 1u);
@@ -437,6 +509,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         const bool valid = jr < p.Co;
         const int o = valid ? __ldg(p.perm + jr) : 0;
         const float bs = (valid && p.bias) ? __ldg(p.bias + jr) : 0.f;
+        const float rs = F16 ? __ldg(p.rscale + jr) : 1.f;  // the layout holds nfb x FB entries
         const int step = pool ? 2 : 1;
         for (int rr = half * step; rr < G::R; rr += 2 * step) {
           const int row = T.r0 + rr;
@@ -444,6 +517,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             float a[16], bb[16];
             tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + cc), a);
             if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + cc), bb);
+            if constexpr (F16) {
+              float a2[16], bb2[16];
+              tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + G::ACC2 + cc), a2);
+              if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + G::ACC2 + cc), bb2);
+              tm_wait_ld();
+#pragma unroll
+              for (int k = 0; k < 16; ++k) {
+                a[k] = fmaf(a2[k], 0x1p-11f, a[k]) * rs;
+                if (pool) bb[k] = fmaf(bb2[k], 0x1p-11f, bb[k]) * rs;
+              }
+            }
             tm_wait_ld();
             // the TMEM loads above are warp-collective; lanes without an output skip only the stores
             if (valid && row < p.H) {
@@ -494,12 +578,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         // a multiply-add and a store.
         constexpr int NR = FB / 32;
         int pm[NR];
-        float bv[NR];
+        float bv[NR], rv[NR];
 #pragma unroll
         for (int k = 0; k < NR; ++k) {
           const int jr = T.fb * FB + 32 * k + lane;
           pm[k] = jr < p.Co ? __ldg(p.perm + jr) : -1;
           bv[k] = (jr < p.Co && p.bias) ? __ldg(p.bias + jr) : 0.f;
+          rv[k] = F16 ? __ldg(p.rscale + jr) : 1.f;  // f16: inverse scale (nfb x FB entries)
         }
         // flattened rows (ORI_PFR): lane j of a segment is row j / TW, column j % TW of it
         const int jl = 32 * q + lane;
@@ -518,6 +603,21 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 #pragma unroll
           for (int jj = half * (FB / 2); jj < (half + 1) * (FB / 2); jj += 16) {
             float a[16], bb[16];
+            if constexpr (F16) {
+              // (acc1 + 2^-11 acc2) times the filter's inverse scale, one row at a time (fewer live
+              // registers); every lane shuffles
+              auto combined = [&](int seg, float (&v)[16]) {
+                float v2[16];
+                tm_ld16(lanebase + (uint32_t)(seg * G::SEGC + jj), v);
+                tm_ld16(lanebase + (uint32_t)(seg * G::SEGC + FB + jj), v2);
+                tm_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 16; ++k)
+                  v[k] = fmaf(v2[k], 0x1p-11f, v[k]) * __shfl_sync(0xffffffffu, rv[(jj + k) >> 5], (jj + k) & 31);
+              };
+              combined(rr, a);
+              if (pool) combined(rr + 1, bb);
+            } else {
             tm_ld16(lanebase + (uint32_t)(rr * G::SEGC + jj), a);
             if (pool) tm_ld16(lanebase + (uint32_t)((rr + 1) * G::SEGC + jj), bb);
             if (G::MRG) {
@@ -532,6 +632,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               }
             }
             tm_wait_ld();
+            }
             // residual (no pool): the 16 skip values are added in a pass of their
             // own, with no store between the loads, so their latencies overlap.
             // The condition is warp-uniform (kernel arguments): every lane takes
@@ -590,8 +691,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 
 template <int ORI, int TW, int FB>
 cudaError_t set_attr() {
-  return cudaFuncSetAttribute(ppconv_tc_kernel<ORI, TW, FB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              Geo<ORI, TW, FB>::SMEM_ALLOC);
+  cudaError_t e = cudaFuncSetAttribute(ppconv_tc_kernel<ORI, TW, FB, false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, Geo<ORI, TW, FB, false>::SMEM_ALLOC);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(ppconv_tc_kernel<ORI, TW, FB, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              Geo<ORI, TW, FB, true>::SMEM_ALLOC);
 }
 
 ppc::DeviceOnce g_attr_once;
@@ -618,30 +722,32 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 std::atomic<EncodeTiledFn> g_encode{nullptr};
 ppc::DeviceOnce g_encode_once;
 
-// 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][8][R+2][TW+8].
-template <int ORI, int TW, int FB>
+// 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][KCH][R+2][TW+8].
+template <int ORI, int TW, int FB, bool F16>
 bool make_xmap(CUtensorMap* m, const TcParams& p) {
-  using G = Geo<ORI, TW, FB>;
+  using G = Geo<ORI, TW, FB, F16>;
   const EncodeTiledFn encode = g_encode.load(std::memory_order_acquire);
   if (!encode) return false;
   const cuuint64_t dims[4] = {(cuuint64_t)p.W, (cuuint64_t)p.H, (cuuint64_t)p.Ci, (cuuint64_t)p.N};
   const cuuint64_t strides[3] = {(cuuint64_t)p.W * 4, (cuuint64_t)p.W * p.H * 4, (cuuint64_t)p.W * p.H * p.Ci * 4};
-  const cuuint32_t box[4] = {(cuuint32_t)G::RAW_W, (cuuint32_t)G::BROWS, (cuuint32_t)KC, 1};
+  const cuuint32_t box[4] = {(cuuint32_t)G::RAW_W, (cuuint32_t)G::BROWS, (cuuint32_t)G::KCH, 1};
   const cuuint32_t estr[4] = {1, 1, 1, 1};
   return encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(p.x), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int ORI, int TW, int FB>
-cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
-  using G = Geo<ORI, TW, FB>;
+template <int ORI, int TW, int FB, bool F16>
+cudaError_t launch_one(const TcParams& p0, cudaStream_t stream, int sms) {
+  using G = Geo<ORI, TW, FB, F16>;
   TcParams p = p0;
+  if ((p.flags & PP_POOL2) && (G::R & 1)) return cudaErrorInvalidValue;  // pooling reads row pairs of a tile
   p.tiles_x = (p.W + TW - 1) / TW;
   p.tiles_y = (p.H + G::R - 1) / G::R;
   CUtensorMap xmap;
   std::memset(&xmap, 0, sizeof(xmap));
-  p.use_tma = ((p.W & 3) == 0 && (reinterpret_cast<uintptr_t>(p.x) & 15) == 0 && make_xmap<ORI, TW, FB>(&xmap, p)) ? 1 : 0;
+  p.use_tma =
+      ((p.W & 3) == 0 && (reinterpret_cast<uintptr_t>(p.x) & 15) == 0 && make_xmap<ORI, TW, FB, F16>(&xmap, p)) ? 1 : 0;
   const int64_t nt = (int64_t)p.tiles_x * p.tiles_y * p.nfb * p.N;
   if (nt > INT32_MAX) return cudaErrorInvalidValue;
   p.ntiles = (int)nt;
@@ -657,7 +763,12 @@ cudaError_t launch(const TcParams& p0, cudaStream_t stream, int sms) {
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB>, p, xmap);
+  return cudaLaunchKernelEx(&cfg, ppconv_tc_kernel<ORI, TW, FB, F16>, p, xmap);
+}
+
+template <int ORI, int TW, int FB>
+cudaError_t launch(const TcParams& p, cudaStream_t stream, int sms, bool f16) {
+  return f16 ? launch_one<ORI, TW, FB, true>(p, stream, sms) : launch_one<ORI, TW, FB, false>(p, stream, sms);
 }
 
 }  // namespace
@@ -742,8 +853,77 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
   return PP_OK;
 }
 
+// The same layer for the fp16 split (PP_PRECISION_F16X3): per (filter block,
+// 16-channel chunk, tap) one tile of 2 FB rows x 16 f16 in the canonical
+// K-major layout, element (row r, channel k) at byte (k / 8) * (2 FB * 16) + r *
+// 16 + (k % 8) * 2, rows 0 .. FB-1 hi = f16(w s) and FB .. 2 FB-1 lo = f16((w s -
+// hi) * 2^11), with s the filter's scale: the power of two that puts its largest
+// kept |w| in [2^13, 2^14).  The input is scaled by xs, the largest power of two
+// with input_bound * xs <= 2^14, so inputs up to twice the bound stay below 2^15
+// (fp16 holds up to 65504).  rscale[j] = 1 / (s_j xs) for reordered filter j
+// (1 / xs for an empty filter and past Co).  Conversions round to nearest.
+pp_status tc_build16(TcLayout* T, const pp_packed* pk, float input_bound, cudaStream_t stream) {
+  const int Co = pk->Co, Ci = pk->Ci, FB = T->FB;
+  if (!(input_bound > 0.f) || !std::isfinite(input_bound)) input_bound = 16384.f;
+  int ex = 0;
+  std::frexp(input_bound, &ex);  // input_bound <= 2^ex
+  const int xs_exp = 14 - ex;
+  const int nch16 = (Ci + 15) / 16;
+  const size_t wtile = (size_t)FB * 16 * 2;
+  const size_t wchunk = NTAP * 2 * wtile;
+  const size_t wbytes = (size_t)T->nfb * nch16 * wchunk;
+  const size_t sbytes = (size_t)T->nfb * FB * 4;
+  std::vector<uint16_t> host(wbytes / 2, 0);
+  std::vector<float> rs((size_t)T->nfb * FB, std::ldexp(1.f, -xs_exp));
+  for (int j = 0; j < Co; ++j) {
+    float mx = 0.f;
+    for (int32_t e = pk->kptr[j]; e < pk->kptr[j + 1]; ++e)
+      for (int q = 0; q < 4; ++q) mx = std::max(mx, std::fabs(pk->kw[(size_t)e * 4 + q]));
+    int we = 0;
+    if (mx > 0.f) std::frexp(mx, &we);  // mx in [2^(we-1), 2^we)
+    const int ws_exp = mx > 0.f ? 14 - we : 0;
+    rs[j] = std::ldexp(1.f, -ws_exp - xs_exp);
+    const int fb = j / FB, f = j % FB;
+    for (int32_t e = pk->kptr[j]; e < pk->kptr[j + 1]; ++e) {
+      const int i = pk->kidx[e], c = i / 16, k = i % 16;
+      const uint8_t* taps = &pk->taps[4 * pk->kpat[e]];
+      for (int q = 0; q < 4; ++q) {
+        const float ws = std::ldexp(pk->kw[(size_t)e * 4 + q], ws_exp);  // exact
+        const __half h = __float2half_rn(ws);
+        const __half l = __float2half_rn((ws - __half2float(h)) * 2048.f);
+        const size_t base = ((size_t)fb * nch16 + c) * wchunk + (size_t)taps[q] * 2 * wtile;
+        const size_t within = (size_t)(k / 8) * (2 * FB * 16) + (size_t)f * 16 + (size_t)(k % 8) * 2;
+        std::memcpy(&host[(base + within) / 2], &h, 2);
+        std::memcpy(&host[(base + within + FB * 16) / 2], &l, 2);
+      }
+    }
+  }
+  void* d = nullptr;
+  if (cudaMalloc(&d, wbytes + sbytes) != cudaSuccess) {
+    cudaGetLastError();
+    return PP_ERR_OOM;
+  }
+  if (cudaMemcpyAsync(d, host.data(), wbytes, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+      cudaMemcpyAsync(static_cast<unsigned char*>(d) + wbytes, rs.data(), sbytes, cudaMemcpyHostToDevice, stream) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess) {
+    cudaFree(d);
+    cudaGetLastError();
+    return PP_ERR_CUDA;
+  }
+  if (T->dmem16) cudaFree(T->dmem16);
+  T->dmem16 = d;
+  T->dbytes16 = wbytes + sbytes;
+  T->a16 = static_cast<const unsigned char*>(d);
+  T->rscale = reinterpret_cast<const float*>(static_cast<unsigned char*>(d) + wbytes);
+  T->nch16 = nch16;
+  T->xscale = std::ldexp(1.f, xs_exp);
+  return PP_OK;
+}
+
 // Geometry the launch will use: orientation and tile width for a map width.
 void tc_geometry(const TcLayout& T, int W, bool pool, int* ori, int* tw) {
+  const bool f16 = T.f16;
   // a pixel-major tile with 128 filters holds one output row (its accumulator
   // row segment is 2 x 128 columns wide), and pooling needs row pairs
   if (T.FB == 64 && !pool && W + 2 <= 64) {
@@ -756,6 +936,9 @@ void tc_geometry(const TcLayout& T, int W, bool pool, int* ori, int* tw) {
   } else {
     *ori = ORI_FP;
     *tw = W <= 16 ? 16 : W <= 32 ? 32 : W <= 64 ? 64 : 128;
+    // f16 filter-major tiles of 128 columns hold one output row (two accumulators per
+    // segment): pooling needs row pairs, so wide pooled maps take 64-column tiles
+    if (f16 && pool && *tw == 128) *tw = 64;
   }
 }
 
@@ -763,11 +946,14 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
                     int W, int flags, cudaStream_t stream) {
   if ((int64_t)M.Co * H * W >= ((int64_t)1 << 31)) return PP_ERR_UNSUPPORTED;  // 32-bit offsets within an image
   if (tc_prepare() != PP_OK) return PP_ERR_CUDA;
+  const bool f16 = T.f16;
   TcParams p;
+  p.rscale = T.rscale;
+  p.xscale = T.xscale;
   p.x = x;
   p.y = y;
   p.skip = (flags & PP_ADD_SKIP) ? skip : nullptr;
-  p.wt = T.a;
+  p.wt = f16 ? T.a16 : T.a;
   p.perm = M.perm;
   p.bias = M.bias;
   p.status = T.status;
@@ -776,7 +962,7 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
   p.Co = M.Co;
   p.H = H;
   p.W = W;
-  p.nch = T.nch;
+  p.nch = f16 ? T.nch16 : T.nch;
   p.nfb = T.nfb;
   p.FB = T.FB;
   p.flags = flags;
@@ -785,18 +971,18 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
   const int sms = device_sms();
   cudaError_t e;
   if (ori == ORI_PF)
-    e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, sms) : launch<ORI_PF, 128, 128>(p, stream, sms);
+    e = T.FB == 64 ? launch<ORI_PF, 128, 64>(p, stream, sms, f16) : launch<ORI_PF, 128, 128>(p, stream, sms, f16);
   else if (ori == ORI_PFR)
-    e = tw == 16 ? launch<ORI_PFR, 16, 64>(p, stream, sms)
-                 : tw == 32 ? launch<ORI_PFR, 32, 64>(p, stream, sms) : launch<ORI_PFR, 64, 64>(p, stream, sms);
+    e = tw == 16 ? launch<ORI_PFR, 16, 64>(p, stream, sms, f16)
+                 : tw == 32 ? launch<ORI_PFR, 32, 64>(p, stream, sms, f16) : launch<ORI_PFR, 64, 64>(p, stream, sms, f16);
   else if (tw == 16)
-    e = launch<ORI_FP, 16, 128>(p, stream, sms);
+    e = launch<ORI_FP, 16, 128>(p, stream, sms, f16);
   else if (tw == 32)
-    e = launch<ORI_FP, 32, 128>(p, stream, sms);
+    e = launch<ORI_FP, 32, 128>(p, stream, sms, f16);
   else if (tw == 64)
-    e = launch<ORI_FP, 64, 128>(p, stream, sms);
+    e = launch<ORI_FP, 64, 128>(p, stream, sms, f16);
   else
-    e = launch<ORI_FP, 128, 128>(p, stream, sms);
+    e = launch<ORI_FP, 128, 128>(p, stream, sms, f16);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return PP_ERR_CUDA;
@@ -807,6 +993,9 @@ pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float
 void tc_free(TcLayout* T) {
   if (T->dmem) cudaFree(T->dmem);
   T->dmem = nullptr;
+  if (T->dmem16) cudaFree(T->dmem16);
+  T->dmem16 = nullptr;
+  T->f16 = false;
   delete T->state;
   T->state = nullptr;
 }

@@ -26,6 +26,17 @@
 // distributed shared memory, adds them in rank order (deterministic), then
 // bias, skip, ReLU, pool, and stores y.  No global workspace is used.
 //
+// Precision: 3xTF32 (as conv_tc.cu), or, for layers set to PP_PRECISION_F16X3,
+// an fp16 split (F16 instantiations): each operand v is held as hi = f16(v) and
+// lo = f16((v - hi) * 2^11), the weights scaled per filter and the input per
+// layer by powers of two so that both stay in fp16's normal range; a chunk is
+// 16 channels (the K of kind::f16) and each tap runs w_hi x_hi into one
+// accumulator and w_lo x_hi + w_hi x_lo into a second one (TMEM columns 128 ..
+// 255 of the buffer), combined in the epilogue as (acc1 + 2^-11 acc2) times the
+// filter's inverse scale.  The dropped lo x lo term and the rounding of the lo
+// parts are each below 2^-22 of |w * x|.  Inputs at or beyond 2^15 after
+// scaling would overflow fp16: the loaders flag them in the device status word.
+//
 // Roles (17 warps, one CTA per SM): warps 0-7 stage the operands, warp 8
 // allocates TMEM and one of its threads issues the MMAs, warps 9-16 are the
 // epilogue (two per TMEM lane quadrant).  Without a split the CTA is persistent
@@ -48,7 +59,8 @@ namespace {
 
 using namespace ppc_ptx;
 
-constexpr int KC = 8;                 // input channels per chunk (MMA K for tf32)
+constexpr int KC = 8;                 // input channels per chunk (MMA K for tf32; 16 for f16)
+constexpr int ACC2 = 128;             // f16: column offset of the second accumulator in a buffer
 constexpr int NTAP = 9;
 constexpr int FB = 128;               // filters per block (MMA M)
 constexpr int NMAX = 256;             // TMEM columns of one accumulator buffer
@@ -58,7 +70,7 @@ constexpr int EPI_WARP0 = 9;          // warps 9-16
 constexpr int NEPI = 256;
 constexpr int NTHREADS = 544;
 constexpr int WMAX = 128;             // widest map handled
-constexpr int W_TILE = FB * KC * 4;   // one tap, hi or lo: 128 x 8 fp32
+constexpr int W_TILE = FB * KC * 4;   // one tap, hi or lo: 128 x 8 fp32 (or 128 x 16 f16)
 constexpr int W_BYTES = NTAP * 2 * W_TILE;
 constexpr int PIX_MAX = 544;          // staged pixels per K half, padding included
 constexpr int IN_MAX = 2 * PIX_MAX * 16;  // largest hi (or lo) operand of one chunk
@@ -71,6 +83,8 @@ static_assert(2 * (W_BYTES + 2 * IN_MAX) <= SMEM_USE, "shared memory plan");
 static_assert(FB * NMAX * 4 <= SMEM_USE, "split reduction buffer");
 
 struct FlatParams {
+  const float* rscale;      // f16: per reordered filter, 1 / (weight scale x input scale)
+  float xscale;             // f16: power of two applied to x before the split
   const float* x;
   float* y;
   const float* skip;
@@ -196,8 +210,10 @@ __device__ __forceinline__ void split_reduce(const FlatParams& p, const Tile& T,
   }
 }
 
-template <bool SPLIT>
+template <bool SPLIT, bool F16>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
+  constexpr int KCH = F16 ? 16 : KC;  // input channels per chunk
+  constexpr int CPH = KCH / 2;         // channels per K half (16 bytes of one pixel row of an operand)
   extern __shared__ unsigned char smem_raw[];
   // Offset from the shared array itself (not an integer round trip), so the
   // compiler keeps every access below in the shared state space.
@@ -217,7 +233,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       if ((i & 255) == 255 && abort_s) return false;
     }
     abort_s = 1;
-    atomicExch(p.status, 1);
+    atomicOr(p.status, ppc::kStatusTimeout);
     return false;
   };
 
@@ -277,7 +293,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       const int pix = it - kh * p.npix;
       const int br = pix / p.bcols, bc = pix - br * p.bcols;
       const bool has = it < 2 * p.npix;
-      roff[b] = has ? (kh * 4 * brows + br) * p.raw_w + bc + 3 : -1;
+      roff[b] = has ? (kh * CPH * brows + br) * p.raw_w + bc + 3 : -1;
       doff[b] = has ? kh * p.npixa + pix : -1;
       rowcol[b] = (kh << 30) | (br << 15) | bc;
     }
@@ -291,7 +307,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       asm volatile(
           "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
           "%4, %5}], [%6];" ::"r"(su32(dst)),
-          "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(-4), "r"(T.r0 - 1), "r"(c * KC), "r"(T.n),
+          "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(-4), "r"(T.r0 - 1), "r"(c * KCH), "r"(T.n),
           "r"(su32(&raw_full[gg & 1]))
           : "memory");
     };
@@ -318,6 +334,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     if (tid == 0 && p.use_tma && p.sep)
       for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + p.raw_off + raw_issued * p.raw_slot);
     bool stop = false;  // identical in every loader thread (decided by group_any)
+    bool range_bad = false;  // f16: an input at or beyond 2^15 after scaling
     for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, tile_index(i));
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
@@ -325,7 +342,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         const int s = g & 1, use = g >> 1;
         // Without a tensor map the chunk's input values are fetched into
         // registers first: that needs no free stage, so it overlaps the wait.
-        float v[ITEMS_MAX][4];
+        float v[ITEMS_MAX][CPH];
         if (!p.use_tma) {
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b) {
@@ -333,8 +350,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             const int r = T.r0 - 1 + br, cc = bc - 1;
             const bool inside = doff[b] >= 0 && (unsigned)r < (unsigned)p.H && (unsigned)cc < (unsigned)p.W;
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const int ch = c * KC + kh * 4 + k;
+            for (int k = 0; k < CPH; ++k) {
+              const int ch = c * KCH + kh * CPH + k;
               v[b][k] = (inside && ch < p.Ci) ? __ldg(xb + ((size_t)ch * p.H + r) * p.W + cc) : 0.f;
             }
           }
@@ -366,7 +383,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b)
 #pragma unroll
-            for (int k = 0; k < 4; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+            for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
           // A ring slot is rewritten next by a tensor-map copy (async proxy): each
           // thread orders its reads of the slot before that copy with a proxy fence.
           if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -380,19 +397,27 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         for (int b = 0; b < ITEMS_MAX; ++b) {
           if (doff[b] >= 0) {
             const int dst = doff[b];
-            float4 h;
-            h.x = tf32_hi(v[b][0]);
-            h.y = tf32_hi(v[b][1]);
-            h.z = tf32_hi(v[b][2]);
-            h.w = tf32_hi(v[b][3]);
-            hi[dst] = h;
-            lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+            if constexpr (F16) {
+              uint4 h, l;
+              range_bad |= split_f16x8(&v[b][0], p.xscale, h, l);
+              reinterpret_cast<uint4*>(hi)[dst] = h;
+              reinterpret_cast<uint4*>(lo)[dst] = l;
+            } else {
+              float4 h;
+              h.x = tf32_hi(v[b][0]);
+              h.y = tf32_hi(v[b][1]);
+              h.z = tf32_hi(v[b][2]);
+              h.w = tf32_hi(v[b][3]);
+              hi[dst] = h;
+              lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
+            }
           }
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         mbar_arrive(su32(&full[s]));
       }
     }
+    if (F16 && range_bad) atomicOr(p.status, ppc::kStatusF16Range);
     if (tid == 0) {
       // No copy may still be writing shared memory when the CTA exits: wait
       // (bounded) for the last copies issued into each stage.
@@ -433,9 +458,16 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             const uint64_t off = (uint64_t)((t / 3) * p.bcols + t % 3);
             const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * W_TILE / 16);
             const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows
-            mma_tf32(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
-            mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
-            mma_tf32(d, whi, xl0 + off, p.idesc, 1u);
+            if (F16) {
+              // acc1 += w_hi x_hi; acc2 += w_lo x_hi + w_hi x_lo (both lo parts scaled by 2^11)
+              mma_f16(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+              mma_f16(d + ACC2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+              mma_f16(d + ACC2, whi, xl0 + off, p.idesc, 1u);
+            } else {
+              mma_tf32(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+              mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
+              mma_tf32(d, whi, xl0 + off, p.idesc, 1u);
+            }
           }
           mma_commit(su32(&empty[s]));
         }
@@ -465,6 +497,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       const Tile T = tile_of(p, tile_index(i));
       const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NMAX);
       const int m = 32 * q + lane;  // filter within the block = TMEM lane
+      // f16: the filter's inverse scale (the layout holds nfb x FB entries, padding included)
+      const float rs = F16 ? __ldg(p.rscale + T.fb * FB + m) : 1.f;
       if (SPLIT) {
         // this CTA's partial tile into its own shared memory (free once the
         // accumulators are ready): row m of [128][ncols + 4], padded so a warp's
@@ -473,11 +507,20 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         // warp-collective loads require)
         float* prow = reinterpret_cast<float*>(smem) + m * (p.ncols + 4);
         for (int cb0 = half * 8; cb0 < p.ncols; cb0 += 64) {
-          float a[4][8];
+          float a[4][8], a2[4][8];
 #pragma unroll
           for (int u = 0; u < 4; ++u)
-            if (cb0 + 16 * u < p.ncols) tm_ld8(lanebase + (uint32_t)(cb0 + 16 * u), a[u]);
+            if (cb0 + 16 * u < p.ncols) {
+              tm_ld8(lanebase + (uint32_t)(cb0 + 16 * u), a[u]);
+              if constexpr (F16) tm_ld8(lanebase + (uint32_t)(ACC2 + cb0 + 16 * u), a2[u]);
+            }
           tm_wait_ld();
+          if constexpr (F16) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int k = 0; k < 8; ++k) a[u][k] = fmaf(a2[u][k], 0x1p-11f, a[u][k]) * rs;
+          }
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
             const int cb = cb0 + 16 * u;
@@ -501,9 +544,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             float* yr = p.y + (plane * p.H + row) * p.W;
             const float* sr = skip ? skip + (plane * p.H + row) * p.W : nullptr;
             for (int cb = 0; cb < p.W; cb += 8) {
-              float a[8];
+              float a[8], a2[8];
               tm_ld8(lanebase + (uint32_t)(rr * p.bcols + cb), a);
+              if constexpr (F16) tm_ld8(lanebase + (uint32_t)(ACC2 + rr * p.bcols + cb), a2);
               tm_wait_ld();
+              if constexpr (F16) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) a[k] = fmaf(a2[k], 0x1p-11f, a[k]) * rs;
+              }
               if (valid) {
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
@@ -530,10 +578,21 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             float* yr = p.y + (plane * Ho + row / 2) * Wo;
             const float* s0 = skip ? skip + (plane * p.H + row) * p.W : nullptr;
             for (int cb = 0; cb < p.W; cb += 8) {
-              float a[8], bb[8];
+              float a[8], bb[8], a2[8], bb2[8];
               tm_ld8(lanebase + (uint32_t)(rr * p.bcols + cb), a);
               tm_ld8(lanebase + (uint32_t)((rr + 1) * p.bcols + cb), bb);
+              if constexpr (F16) {
+                tm_ld8(lanebase + (uint32_t)(ACC2 + rr * p.bcols + cb), a2);
+                tm_ld8(lanebase + (uint32_t)(ACC2 + (rr + 1) * p.bcols + cb), bb2);
+              }
               tm_wait_ld();
+              if constexpr (F16) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                  a[k] = fmaf(a2[k], 0x1p-11f, a[k]) * rs;
+                  bb[k] = fmaf(bb2[k], 0x1p-11f, bb[k]) * rs;
+                }
+              }
               if (valid) {
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
@@ -617,13 +676,22 @@ cudaError_t init_device(int dev) {
   DeviceState& D = g_dev[dev];
   cudaError_t e = cudaDeviceGetAttribute(&D.sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(ppconv_tcf_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
-          cudaSuccess ||
-      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
-          cudaSuccess)
+  if ((e = cudaFuncSetAttribute(ppconv_tcf_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SMEM_ALLOC)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SMEM_ALLOC)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SMEM_ALLOC)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SMEM_ALLOC)) != cudaSuccess)
     return e;
-  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
-    cudaGetLastError();  // then only portable sizes (up to 8) can be used
+  // then only portable sizes (up to 8) can be used
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+      cudaSuccess)
+    cudaGetLastError();
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+      cudaSuccess)
+    cudaGetLastError();
   for (int s = 2; s <= MAX_SPLIT; s *= 2) {
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute at[1];
@@ -637,7 +705,8 @@ cudaError_t init_device(int dev) {
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, ppconv_tcf_kernel<true>, &cfg) != cudaSuccess) {
+    // both precisions launch 544 threads, one CTA per SM, with the same shared memory
+    if (cudaOccupancyMaxActiveClusters(&n, ppconv_tcf_kernel<true, false>, &cfg) != cudaSuccess) {
       cudaGetLastError();
       n = 0;
     }
@@ -677,11 +746,15 @@ struct FlatGeo {
 // cycle; and clusters beyond those co-resident on the GPU run in later waves.
 // Every geometry the kernel can run for this shape, best first by the model;
 // fills up to maxn entries and returns how many.
+// f16: nch counts 16-channel chunks, an accumulator is at most 128 columns (the
+// second one follows it in the same buffer) and the input box holds 16 channels.
 int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
-                    FlatGeo* out, int maxn) {
+                    FlatGeo* out, int maxn, bool f16) {
   if (W < 1 || W > WMAX || H < 1 || maxn < 1) return 0;
   const int bcols = (W + 2 + 7) / 8 * 8;
-  const int rmax = NMAX / bcols;
+  const int nmax = f16 ? ACC2 : NMAX;
+  const int kch = f16 ? 16 : KC;
+  const int rmax = nmax / bcols;
   if (rmax < 1 || (pool && rmax < 2)) return 0;
   int n = 0;
   for (int r0 = rmax; r0 >= 1; --r0) {
@@ -701,7 +774,7 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
     G.npix = (R + 2) * bcols;
     G.npixa = G.npix + 16;
     G.raw_w = bcols + 4;
-    G.raw_bytes = KC * (R + 2) * G.raw_w * 4;
+    G.raw_bytes = kch * (R + 2) * G.raw_w * 4;
     G.tiles_y = ty;
     const int64_t nt = (int64_t)ty * nfb * N;
     const int in_bytes = (2 * G.npixa * 16 + 127) / 128 * 128;
@@ -711,7 +784,7 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
     if (!G.sep) G.stage = W_BYTES + in_bytes + std::max(in_bytes, G.raw_slot);  // the box lands in lo
     G.lo_off = W_BYTES + in_bytes;
     G.raw_off = 2 * G.stage;
-    if (G.npixa > PIX_MAX || 2 * G.stage > SMEM_USE || G.ncols > NMAX || nt > INT32_MAX / MAX_SPLIT) continue;
+    if (G.npixa > PIX_MAX || 2 * G.stage > SMEM_USE || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
     G.ntiles = (int)nt;
     const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
     const double per_chunk = std::max(std::max(mma, W_BYTES / 48.0), 1500.0);
@@ -745,14 +818,15 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
 }
 
 bool flat_geometry(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
-                   FlatGeo* out) {
-  return flat_candidates(N, H, W, nch, nfb, pool, allow_split, D, out, 1) == 1;
+                   FlatGeo* out, bool f16) {
+  return flat_candidates(N, H, W, nch, nfb, pool, allow_split, D, out, 1, f16) == 1;
 }
 
 // The geometry (R, split) for this shape if the model can run it.
-bool flat_pick(int N, int H, int W, int nch, int nfb, bool pool, const DeviceState& D, int R, int S, FlatGeo* out) {
+bool flat_pick(int N, int H, int W, int nch, int nfb, bool pool, const DeviceState& D, int R, int S, FlatGeo* out,
+               bool f16) {
   FlatGeo all[160];
-  const int n = flat_candidates(N, H, W, nch, nfb, pool, true, D, all, 160);
+  const int n = flat_candidates(N, H, W, nch, nfb, pool, true, D, all, 160, f16);
   for (int k = 0; k < n; ++k)
     if (all[k].R == R && all[k].split == S) {
       *out = all[k];
@@ -765,7 +839,7 @@ bool flat_pick(int N, int H, int W, int nch, int nfb, bool pool, const DeviceSta
 bool pinned_geometry(const ppc::TcLayout& T, int N, int H, int W, int flags, const DeviceState& D, FlatGeo* out) {
   const ppc::TcState* st = T.state;
   if (!st || st->R <= 0 || st->key[0] != N || st->key[1] != H || st->key[2] != W || st->key[3] != flags) return false;
-  return flat_pick(N, H, W, T.nch, T.nfb, flags & PP_POOL2, D, st->R, st->S, out);
+  return flat_pick(N, H, W, T.f16 ? T.nch16 : T.nch, T.nfb, flags & PP_POOL2, D, st->R, st->S, out, T.f16);
 }
 
 pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
@@ -782,7 +856,8 @@ pp_status tcf_launch(const TcLayout& T, const LayerMeta& M, const float* x, floa
   if (!D) return PP_ERR_CUDA;
   const bool pool = flags & PP_POOL2;
   FlatGeo G;
-  if (!pinned_geometry(T, N, H, W, flags, *D, &G) && !flat_geometry(N, H, W, T.nch, T.nfb, pool, true, *D, &G))
+  if (!pinned_geometry(T, N, H, W, flags, *D, &G) &&
+      !flat_geometry(N, H, W, T.f16 ? T.nch16 : T.nch, T.nfb, pool, true, *D, &G, T.f16))
     return PP_ERR_UNSUPPORTED;
   return launch_geo(G, *D, T, M, x, y, skip, N, H, W, flags, stream);
 }
@@ -794,11 +869,15 @@ namespace {
 pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLayout& T, const ppc::LayerMeta& M,
                      const float* x, float* y, const float* skip, int N, int H, int W, int flags, cudaStream_t stream) {
   const DeviceState* D = &Dref;
+  const bool f16 = T.f16;
+  const int kch = f16 ? 16 : KC;
   FlatParams p;
+  p.rscale = T.rscale;
+  p.xscale = T.xscale;
   p.x = x;
   p.y = y;
   p.skip = (flags & PP_ADD_SKIP) ? skip : nullptr;
-  p.wt = T.a;
+  p.wt = f16 ? T.a16 : T.a;
   p.perm = M.perm;
   p.bias = M.bias;
   p.status = T.status;
@@ -807,7 +886,7 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.Co = M.Co;
   p.H = H;
   p.W = W;
-  p.nch = T.nch;
+  p.nch = f16 ? T.nch16 : T.nch;
   p.nfb = T.nfb;
   p.flags = flags;
   p.bcols = G.bcols;
@@ -825,7 +904,7 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.tiles_y = G.tiles_y;
   p.ntiles = G.ntiles;
   p.split = G.split;
-  p.idesc = idesc_tf32(FB, G.ncols);
+  p.idesc = f16 ? idesc_f16(FB, G.ncols) : idesc_tf32(FB, G.ncols);
   CUtensorMap xmap;
   std::memset(&xmap, 0, sizeof(xmap));
   p.use_tma = 0;
@@ -833,7 +912,7 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
     // 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][8][R+2][BCOLS+4]
     const cuuint64_t dims[4] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)M.Ci, (cuuint64_t)N};
     const cuuint64_t strides[3] = {(cuuint64_t)W * 4, (cuuint64_t)W * H * 4, (cuuint64_t)W * H * M.Ci * 4};
-    const cuuint32_t box[4] = {(cuuint32_t)G.raw_w, (cuuint32_t)(G.R + 2), (cuuint32_t)KC, 1};
+    const cuuint32_t box[4] = {(cuuint32_t)G.raw_w, (cuuint32_t)(G.R + 2), (cuuint32_t)kch, 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     p.use_tma = D->encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(x), dims, strides, box, estr,
                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
@@ -860,10 +939,12 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
     at[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
     cfg.gridDim = dim3((unsigned)(G.ntiles * G.split));
-    e = cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true>, p, xmap);
+    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, true>, p, xmap)
+            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, false>, p, xmap);
   } else {
     cfg.gridDim = dim3((unsigned)std::min(G.ntiles, D->sms));
-    e = cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false>, p, xmap);
+    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false, true>, p, xmap)
+            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false, false>, p, xmap);
   }
   if (e != cudaSuccess) {
     cudaGetLastError();
@@ -881,7 +962,8 @@ int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, 
   DeviceState* D = prepare();
   if (!D) return 0;
   FlatGeo G[16];
-  const int n = flat_candidates(N, H, W, T.nch, T.nfb, flags & PP_POOL2, true, *D, G, std::min(maxn, 16));
+  const int n = flat_candidates(N, H, W, T.f16 ? T.nch16 : T.nch, T.nfb, flags & PP_POOL2, true, *D, G,
+                                std::min(maxn, 16), T.f16);
   for (int k = 0; k < n; ++k) {
     R[k] = G[k].R;
     S[k] = G[k].split;
@@ -893,7 +975,7 @@ bool tcf_can_run(const TcLayout& T, int N, int H, int W, int flags, int R, int S
   if (T.FB != FB) return false;
   DeviceState* D = prepare();
   FlatGeo G;
-  return D && flat_pick(N, H, W, T.nch, T.nfb, flags & PP_POOL2, *D, R, S, &G);
+  return D && flat_pick(N, H, W, T.f16 ? T.nch16 : T.nch, T.nfb, flags & PP_POOL2, *D, R, S, &G, T.f16);
 }
 
 void tcf_pinned(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S) {

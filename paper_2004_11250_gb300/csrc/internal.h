@@ -84,21 +84,36 @@ struct TcState {
 };
 
 // Dense per-tap tf32 hi/lo weight tiles of the tensor-core kernels (conv_tc.cu,
-// conv_tcf.cu).
+// conv_tcf.cu), and, once the layer's precision is PP_PRECISION_F16X3, their
+// f16 counterpart.
 struct TcLayout {
   int FB = 128, nfb = 0, nch = 0;
   void* dmem = nullptr;
   size_t dbytes = 0;
   const unsigned char* a = nullptr;
-  int* status = nullptr;        // device word, nonzero after a timed-out wait
+  int* status = nullptr;        // device word: bit 0 a timed-out wait, bit 1 an input out of the f16 range
   TcState* state = nullptr;  // owned; see tc_free
+  // fp16 split: [nfb][nch16][9][2 FB x 16 f16] tiles (hi rows, then lo rows scaled by 2^11) and, per
+  // reordered filter, 1 / (its weight scale x the input scale), a power of two
+  bool f16 = false;             // launches run the f16 instantiations
+  int nch16 = 0;                // 16-channel chunks
+  float xscale = 1.f;           // power of two applied to x before the split
+  void* dmem16 = nullptr;
+  size_t dbytes16 = 0;
+  const unsigned char* a16 = nullptr;
+  const float* rscale = nullptr;
 };
+// Device status bits of a tensor-core layer.
+constexpr int kStatusTimeout = 1;
+constexpr int kStatusF16Range = 2;
 
 pp_status tc_prepare();
 pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream);
 pp_status tc_launch(const TcLayout& T, const LayerMeta& M, const float* x, float* y, const float* skip, int N,
                     int H, int W, int flags, cudaStream_t stream);
 pp_status tc_status(const TcLayout& T, int* device_error);
+// Build the f16 tiles and scales (precision PP_PRECISION_F16X3) for inputs bounded by input_bound.
+pp_status tc_build16(TcLayout* T, const pp_packed* pk, float input_bound, cudaStream_t stream);
 void tc_free(TcLayout* T);
 // Flat variant (maps up to 128 pixels wide, 128-filter blocks); returns
 // PP_ERR_UNSUPPORTED for shapes it does not handle.

@@ -46,6 +46,12 @@ PP_PROBE_FFMA = 0
 PP_PROBE_MMA_TF32 = 1
 PP_PROBE_MMA_F16 = 2
 
+PP_PRECISION_TF32X3 = 0
+PP_PRECISION_F16X3 = 1
+
+PP_STATUS_TIMEOUT = 1
+PP_STATUS_F16_RANGE = 2
+
 PP_ADD_SKIP = 1
 PP_RELU = 2
 PP_POOL2 = 4
@@ -70,6 +76,8 @@ _SIGS = {
     "pp_conv_forward_noalloc": ([_P, _P, _P, _P, _I, _I, _I, _I, _P], _I),
     "pp_layer_set_kernel": ([_P, _I], _I),
     "pp_layer_set_output_order": ([_P, _P, _P], _I),
+    "pp_layer_set_precision": ([_P, _I, ctypes.c_float, _P], _I),
+    "pp_layer_precision": ([_P, _P, _P], _I),
     "pp_permute_input_channels": ([_P, _P, _P, _I, _I, _P, _P, _P, _P], _I),
     "pp_layer_kernel": ([_P, _P], _I),
     "pp_layer_device_status": ([_P, _P], _I),
@@ -272,6 +280,18 @@ def pp_layer_set_output_order(layer, order=None, stream=None):
     """order[o] = output channel of original filter o (None: original order); see the header."""
     o = _host(order, np.int32)
     _check(lib.pp_layer_set_output_order(layer, _hp(o), _stream(stream)), "pp_layer_set_output_order")
+
+
+def pp_layer_set_precision(layer, precision: int, input_bound: float = 0.0, stream=None):
+    """PP_PRECISION_TF32X3 or PP_PRECISION_F16X3 for the tensor-core kernels (see the header)."""
+    _check(lib.pp_layer_set_precision(layer, precision, float(input_bound), _stream(stream)), "pp_layer_set_precision")
+
+
+def pp_layer_precision(layer):
+    """(precision, input scale)."""
+    p, sc = _I(), ctypes.c_float()
+    _check(lib.pp_layer_precision(layer, ctypes.byref(p), ctypes.byref(sc)), "pp_layer_precision")
+    return p.value, sc.value
 
 
 def pp_layer_kernel(layer) -> int:

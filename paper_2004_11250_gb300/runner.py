@@ -33,7 +33,8 @@ class DeviceLayer:
     in_layout[c]); the weights' input channels are permuted to match before packing.  None = original order.
     """
 
-    def __init__(self, layer, stream=None, in_layout: Optional[np.ndarray] = None):
+    def __init__(self, layer, stream=None, in_layout: Optional[np.ndarray] = None, precision: int = 0,
+                 input_bound: float = 0.0):
         self.spec = layer
         self.packed = None
         self.dense = isinstance(layer, synth.DenseLayer)
@@ -46,6 +47,8 @@ class DeviceLayer:
         else:
             self.packed = pp.pp_pack_layer(w, mask, layer.taps)
             self.handle = pp.pp_layer_create(self.packed, layer.bias, stream)
+            if precision != pp.PP_PRECISION_TF32X3 and layer.Ci >= 8:  # layers with a tensor-core layout
+                pp.pp_layer_set_precision(self.handle, precision, input_bound, stream)
 
     def perm(self) -> np.ndarray:
         return pp.pp_packed_arrays(self.packed)["perm"].copy()
@@ -94,9 +97,13 @@ class DeviceNet:
     input channels permuted to match, so activations between layers stay in reordered order.  Activations
     tied to the network input or output, to a dense layer, or to such a group through a skip keep the
     original order; an op adding a skip stores its output in the skip's order.
+
+    precision / input_bound: the tensor-core arithmetic of every pruned layer that has a tensor-core
+    layout (pp_layer_set_precision).
     """
 
-    def __init__(self, spec: synth.Net, use_graph: bool = True, stream=None, fold_perm: bool = False):
+    def __init__(self, spec: synth.Net, use_graph: bool = True, stream=None, fold_perm: bool = False,
+                 precision: int = 0, input_bound: float = 0.0):
         self.spec = spec
         N, C, H, W = spec.x.shape
         self.layers: List[DeviceLayer] = []
@@ -105,7 +112,7 @@ class DeviceNet:
         for k, op in enumerate(spec.ops):
             lay_in = self.layouts[k]
             ident = bool((lay_in == np.arange(len(lay_in))).all())
-            L = DeviceLayer(op.layer, stream, None if ident else lay_in)
+            L = DeviceLayer(op.layer, stream, None if ident else lay_in, precision, input_bound)
             Co = op.layer.Co
             if keep_orig[k + 1]:
                 lay_out = np.arange(Co, dtype=np.int32)

@@ -35,8 +35,8 @@ def dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def run_layer(pp, runner, layer, x, skip=None, relu=False, pool=False, kernel=None):
-    L = runner.DeviceLayer(layer)
+def run_layer(pp, runner, layer, x, skip=None, relu=False, pool=False, kernel=None, precision=0):
+    L = runner.DeviceLayer(layer, precision=precision)
     try:
         if kernel is not None:
             pp.pp_layer_set_kernel(L.handle, kernel)
@@ -46,6 +46,8 @@ def run_layer(pp, runner, layer, x, skip=None, relu=False, pool=False, kernel=No
         flags = (pp.PP_ADD_SKIP if skip is not None else 0) | (pp.PP_RELU if relu else 0) | (pp.PP_POOL2 if pool else 0)
         L.forward(dev(x), y, None if skip is None else dev(skip), N, H, W, flags, torch.cuda.current_stream())
         torch.cuda.synchronize()
+        if not L.dense:
+            assert pp.pp_layer_device_status(L.handle) == 0
         return y.cpu().numpy()
     finally:
         L.close()
@@ -495,12 +497,12 @@ def test_cfg0_full(pp, runner, oracle_mod):
     check_within(g, y, s, "cfg0")
 
 
-def layerwise_check(pp, runner, oracle_mod, net, check_net=True, fold_perm=False):
+def layerwise_check(pp, runner, oracle_mod, net, check_net=True, fold_perm=False, precision=0):
     """Run a network op by op on the GPU and check every output of every op against the oracle
     evaluated on the GPU's own input to that op (rearranged into the original channel order when the
     filter reorder is folded into the next layer); then check the executor reproduces the op-by-op
     result bit for bit (direct launches and CUDA-graph replay) and the host-buffer path too."""
-    dn = runner.DeviceNet(net, use_graph=True, fold_perm=fold_perm)
+    dn = runner.DeviceNet(net, use_graph=True, fold_perm=fold_perm, precision=precision)
     try:
         x = dev(net.x)
         acts = dn.run_layerwise(x)
@@ -740,3 +742,163 @@ def test_peak_probes(pp):
     t16, m16, _ = pp.pp_peak_probe(pp.PP_PROBE_MMA_F16, 1 << 12)
     assert t32 > 5 * tf and t16 > 1.3 * t32, (tf, t32, t16)
     assert 300 < m32 < 2500 and 300 < m16 < 2500
+
+
+# ----------------------------------------------------------------------------- fp16 split (PP_PRECISION_F16X3)
+
+F16 = 1  # PP_PRECISION_F16X3
+
+
+@pytest.mark.parametrize("case", [c for c in SMALL if c[1] >= 8])
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+@pytest.mark.parametrize("kernel", ["TC", "TC_FLAT"])
+def test_f16_small(pp, runner, oracle_mod, case, flags, kernel):
+    """The fp16-split arithmetic on every small case with at least 8 input channels, both tensor-core
+    kernels (layers with at most 64 filters run the row-tiled kernel for TC_FLAT), every output."""
+    N, Ci, Co, H, W, P, ring, keep = case
+    if flags == "pool_relu" and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(13 * sum(case[:5]) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=P, keep=keep, ring=ring)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    k = getattr(pp, "PP_KERNEL_" + kernel) if (kernel == "TC" or Co > 64) else pp.PP_KERNEL_TC
+    g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=k, precision=F16)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
+    check_within(g, y, s, f"f16 {kernel} {case} {flags}")
+
+
+@pytest.mark.parametrize("case", FLAT_CASES)
+@pytest.mark.parametrize("flags", ["none", "skip_pool_relu"])
+def test_f16_flat_kernel(pp, runner, oracle_mod, case, flags):
+    N, Ci, Co, H, W = case
+    pool = "pool" in flags and H % 2 == 0 and W % 2 == 0
+    rng = np.random.default_rng(17 * sum(case) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.45, ring=sum(case) % 2 == 0)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if "skip" in flags else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", pool, kernel=pp.PP_KERNEL_TC_FLAT, precision=F16)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", pool)
+    check_within(g, y, s, f"f16 flat {case} {flags}")
+
+
+@pytest.mark.parametrize("shape", [(1, 40, 130, 7, 100), (2, 16, 200, 4, 144), (1, 24, 64, 6, 160)] + PFR_CASES)
+@pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
+def test_f16_row_tiled(pp, runner, oracle_mod, shape, flags):
+    """Row-tiled kernel under f16: pixel-major (128- and 64-filter blocks), flattened rows, filter-major."""
+    N, Ci, Co, H, W = shape
+    pool = flags == "pool_relu"
+    if pool and (H % 2 or W % 2):
+        pytest.skip("pool needs even sizes")
+    rng = np.random.default_rng(19 * sum(shape) + len(flags))
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.4)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if flags == "skip_relu" else None
+    g = run_layer(pp, runner, L, x, skip, flags != "none", pool, kernel=pp.PP_KERNEL_TC, precision=F16)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", pool)
+    check_within(g, y, s, f"f16 row-tiled {shape} {flags}")
+
+
+@pytest.mark.parametrize("shape,kernel", [((1, 136, 130, 28, 28), "TC_FLAT"), ((6, 40, 200, 14, 14), "TC_FLAT"),
+                                          ((1, 40, 64, 20, 150), "TC"), ((2, 24, 130, 9, 40), "TC")])
+def test_f16_integer_bit_exact(pp, runner, oracle_mod, shape, kernel):
+    """Integer weights in [-4, 4] and inputs in [-8, 8]: f16 holds them exactly (lo parts zero), the
+    power-of-two scales are exact and every partial sum is an exact fp32 value, so the result equals
+    the oracle bit for bit."""
+    N, Ci, Co, H, W = shape
+    rng = np.random.default_rng(Co + W + 1)
+    L = synth.integer_layer(rng, Co, Ci, synth.ring8_patterns(), 0.5)
+    x = rng.integers(-8, 9, (N, Ci, H, W)).astype(np.float32)
+    g = run_layer(pp, runner, L, x, None, True, False, kernel=getattr(pp, "PP_KERNEL_" + kernel), precision=F16)
+    y, _ = oracle_layer_full(oracle_mod, L, x, None, True, False)
+    assert (g.astype(np.float64) == y).all()
+
+
+@pytest.mark.parametrize("shape,kernel", [((12, 256, 256, 56, 56), "TC"), ((8, 64, 64, 128, 128), "TC"),
+                                          ((12, 256, 256, 56, 56), "TC_FLAT"), ((1, 512, 512, 28, 28), "TC_FLAT"),
+                                          ((1, 512, 512, 14, 14), "TC_FLAT"), ((2, 128, 128, 112, 112), "TC_FLAT")])
+def test_f16_repeatable_multi_tile(pp, runner, oracle_mod, shape, kernel):
+    """As test_tensor_core_repeatable_multi_tile, under f16: five runs bit for bit equal, every output
+    within the bound, device status clear."""
+    N, Ci, Co, H, W = shape
+    rng = np.random.default_rng(Ci + W + 2)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=1.0)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    dl = runner.DeviceLayer(L, precision=F16)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, getattr(pp, "PP_KERNEL_" + kernel))
+        xd = dev(x)
+        outs = []
+        for _ in range(5):
+            y = torch.full((N, Co, H, W), float("nan"), device="cuda")
+            dl.forward(xd, y, None, N, H, W, 0, torch.cuda.current_stream())
+            outs.append(y)
+        torch.cuda.synchronize()
+        for k in range(1, 5):
+            assert torch.equal(outs[0], outs[k]), f"run {k} differs from run 0"
+        assert pp.pp_layer_device_status(dl.handle) == 0
+        yr, s = oracle_layer_full(oracle_mod, L, x)
+        check_within(outs[0].cpu().numpy(), yr, s, f"f16 multi-tile {shape}")
+    finally:
+        dl.close()
+
+
+@pytest.mark.parametrize("name", ["vgg16", "style", "vdsr"])
+def test_f16_workloads(pp, runner, oracle_mod, name):
+    """The three networks under f16 (every pruned layer with a tensor-core layout), every output of
+    every op against the oracle on the GPU's own input, executor replays bit for bit."""
+    net = {"vgg16": synth.cfg1_vgg16, "style": synth.cfg2_style, "vdsr": synth.cfg3_vdsr}[name]()
+    assert layerwise_check(pp, runner, oracle_mod, net, precision=F16) < 1e-5
+
+
+@pytest.mark.parametrize("point", synth.cfg4_points())
+def test_f16_sweep_point(pp, runner, oracle_mod, point):
+    """Every output of every sweep point under f16, at the kernel autotuning picks for its shape."""
+    C, P, keep = point
+    net = synth.cfg4_point(C, P, keep)
+    L = net.ops[0].layer
+    N, _, H, W = net.x.shape
+    dl = runner.DeviceLayer(L, precision=F16)
+    try:
+        pp.pp_layer_autotune(dl.handle, N, H, W, 0, torch.cuda.current_stream())
+        y = torch.full((N, C, H, W), float("nan"), device="cuda")
+        dl.forward(dev(net.x), y, None, N, H, W, 0, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        assert pp.pp_layer_device_status(dl.handle) == 0
+        g = y.cpu().numpy()
+    finally:
+        dl.close()
+    yr, s = oracle_layer_full(oracle_mod, L, net.x)
+    check_within(g, yr, s, f"f16 sweep {point}")
+
+
+@pytest.mark.parametrize("kernel", ["TC", "TC_FLAT"])
+def test_f16_input_range(pp, runner, oracle_mod, kernel):
+    """An input at 2^15 or beyond (after the layer's input scale) is flagged in the device status word
+    (bit 1), not silently wrong; with a bound that covers it (input scale 2^-3 for a bound of 1e5) the
+    same input is within the error bound; the precision and scale read back."""
+    rng = np.random.default_rng(5)
+    Co, Ci, N, H, W = 136, 16, 1, 12, 20
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.5)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    x[0, 3, 5, 7] = 40000.0
+    dl = runner.DeviceLayer(L, precision=F16)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, getattr(pp, "PP_KERNEL_" + kernel))
+        assert pp.pp_layer_precision(dl.handle) == (F16, 1.0)
+        y = torch.empty((N, Co, H, W), device="cuda")
+        dl.forward(dev(x), y, None, N, H, W, 0, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        assert pp.pp_layer_device_status(dl.handle) == pp.PP_STATUS_F16_RANGE
+        assert pp.pp_layer_device_status(dl.handle) == 0  # cleared by the read
+        pp.pp_layer_set_precision(dl.handle, F16, 1e5)
+        assert pp.pp_layer_precision(dl.handle) == (F16, 2.0 ** -3)
+        dl.forward(dev(x), y, None, N, H, W, 0, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        assert pp.pp_layer_device_status(dl.handle) == 0
+        yr, s = oracle_layer_full(oracle_mod, L, x)
+        check_within(y.cpu().numpy(), yr, s, f"f16 {kernel} with a bound of 1e5")
+        pp.pp_layer_set_precision(dl.handle, 0)
+        assert pp.pp_layer_precision(dl.handle) == (0, 1.0)
+    finally:
+        dl.close()
