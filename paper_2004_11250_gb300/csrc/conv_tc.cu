@@ -131,7 +131,9 @@ struct Geo {
   // pixels past the staged tile (junk columns only); 16 pixels of slack
   static constexpr int NPIXA = ORI == ORI_PFR ? NPIX + 16 : NPIX;
   static constexpr int IN_HALF = NPIXA * 16;              // one K half (4 channels) of hi or lo
-  static constexpr int IN_BYTES = 2 * IN_HALF;            // hi or lo, 8 channels
+  // hi or lo operand of a chunk; a multiple of 128 bytes, so the lo area (where the input box lands
+  // when it has no slot of its own) starts where a tensor-map copy may write
+  static constexpr int IN_BYTES = (2 * IN_HALF + 127) / 128 * 128;
   // tensor-map box width: columns c0-4 .. (staged column bc is box column bc + 3),
   // a multiple of 4 so each box row is whole 16-byte units
   static constexpr int RAW_W = (BCOLS + 3 + 3) / 4 * 4;
@@ -149,6 +151,8 @@ struct Geo {
   static constexpr int SMEM_ALLOC = 2 * STAGE + (SEP ? 2 * RAW : 0) + 1024;
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
   static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
+  static_assert(W_BYTES % 128 == 0 && IN_BYTES % 128 == 0 && RAW % 128 == 0 && STAGE % 128 == 0,
+                "tensor-map copies need 128-byte aligned shared-memory destinations");
   static constexpr uint32_t IDESC = F16 ? (ORI == ORI_FP ? idesc_f16(128, TW) : idesc_f16(128, FB))
                                         : (ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB));
   static constexpr uint32_t IDESC2 = F16 ? idesc_f16(128, 2 * FB) : idesc_tf32(128, 2 * FB);  // MRG: [w_hi | w_lo]
@@ -442,7 +446,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           // lies below 256 KB, so moving an operand is one add to the descriptor.
           const uint64_t w0 = smem_desc(su32(st), G::WLBO);
           const uint64_t xh0 = smem_desc(su32(st + G::W_BYTES), G::IN_HALF);
-          const uint64_t xl0 = smem_desc(su32(st + G::W_BYTES + G::IN_HALF * 2), G::IN_HALF);
+          const uint64_t xl0 = smem_desc(su32(st + G::W_BYTES + G::IN_BYTES), G::IN_HALF);
           const uint32_t acc0 = c == 0 ? 0u : 1u;  // the tile's first chunk overwrites the accumulators
 #pragma unroll
           for (int t = 0; t < NTAP; ++t) {
