@@ -870,7 +870,8 @@ pp_status tc_build16(TcLayout* T, const pp_packed* pk, float input_bound, cudaSt
   const int Co = pk->Co, Ci = pk->Ci, FB = T->FB;
   if (!(input_bound > 0.f) || !std::isfinite(input_bound)) input_bound = 16384.f;
   int ex = 0;
-  std::frexp(input_bound, &ex);  // input_bound <= 2^ex
+  const float m = std::frexp(input_bound, &ex);  // input_bound = m 2^ex, m in [0.5, 1)
+  if (m == 0.5f) --ex;                             // ex = ceil(log2(input_bound))
   const int xs_exp = 14 - ex;
   const int nch16 = (Ci + 15) / 16;
   const size_t wtile = (size_t)FB * 16 * 2;
