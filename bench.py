@@ -103,7 +103,24 @@ def workload(name: str):
     if name.startswith("sweep:"):  # sweep:C:P:keep, one point of the throughput sweep
         C, P, keep = name.split(":")[1:]
         return synth.cfg4_point(int(C), int(P), float(keep))
+    if name.startswith("op:"):  # op:<workload>:<k>, op k of a network alone (for profiling one layer)
+        base, k = name.split(":")[1:]
+        return single_op(workload(base), int(k))
     raise ValueError(name)
+
+
+def single_op(spec, k):
+    """Op k of a network as a one-op network: same layer, flags and input shape; the input is seeded
+    U(0, 1) (a ReLU network's activations are non-negative) and a skip, if any, is dropped."""
+    from paper_2004_11250_gb300 import synth
+    N, C, H, W = spec.x.shape
+    for op in spec.ops[:k]:
+        C = op.layer.Co
+        if op.pool:
+            H, W = H // 2, W // 2
+    op = spec.ops[k]
+    x = np.random.default_rng(k).uniform(0, 1, size=(N, C, H, W)).astype(np.float32)
+    return synth.Net(f"{spec.name}_op{k}", x, [synth.Op(op.layer, relu=op.relu, pool=op.pool)])
 
 
 def op_shapes(spec):
@@ -508,6 +525,9 @@ def metric_name(w):
     if w.startswith("sweep:"):
         C, P, keep = w.split(":")[1:]
         name = f"sweep point 8x{C}x56x56, C_in = C_out = {C}, {P} patterns, keep {keep}"
+    elif w.startswith("op:"):
+        base, k = w.split(":")[1:]
+        name = f"op {k} of the {names[base]} alone"
     else:
         name = names[w]
     return f"effective GFLOP/s (surviving MACs), {name}, fp32"
@@ -531,7 +551,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="vgg16",
-                    help="vgg16 (default), single, style, vdsr, or sweep:C:P:keep (one point of the sweep)")
+                    help="vgg16 (default), single, style, vdsr, sweep:C:P:keep (one point of the sweep), or "
+                         "op:<workload>:<k> (op k of a network alone, to profile one layer)")
     ap.add_argument("--precision", default="tf32x3", choices=["tf32x3", "f16x3"],
                     help="arithmetic of the tensor-core kernels for the timed frames (pp_layer_set_precision)")
     ap.add_argument("--fold-perm", action="store_true",

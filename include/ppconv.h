@@ -227,9 +227,10 @@ pp_status pp_layer_set_output_order(pp_layer* layer, const int32_t* order, void*
  *       fp16's subnormal spacing adds at most 2^-36 / s_x per unit of |w|, so
  *       the bound holds unless an output's whole receptive field is tiny
  *       (mean |x| below ~1e-6 / s_x) yet not zero.  Inputs must satisfy
- *       |x_s| < 2^15 (|x| < 2 * input_bound at least); a launch that meets a
- *       larger one sets bit 1 of the layer's device status word and its
- *       output is invalid.  input_bound <= 0 means 16384 (s_x = 1).
+ *       |x_s| < 65504, fp16's largest value (|x| < 4 * input_bound at least);
+ *       a launch that meets a larger input, or one that is not finite, sets
+ *       bit 1 of the layer's device status word and its output is invalid.
+ *       input_bound <= 0 means 16384 (s_x = 1).
  * Switching to PP_PRECISION_F16X3 builds the f16 weight layout (half the
  * bytes of the tf32 one) from a host copy of the packed layer, synchronously
  * on stream; a CUDA graph captured before keeps the old arithmetic.
@@ -308,8 +309,8 @@ pp_status pp_layer_pin_flat_geometry(pp_layer* layer, int N, int H, int W, int f
 /* Synchronous: *device_error = 0 unless a launch of this layer's tensor-core
  * kernels met an error since the last read, and its output is then invalid:
  * bit 0 (value 1) a bounded wait gave up; bit 1 (value 2) under
- * PP_PRECISION_F16X3 an input was at or beyond 2^15 after the layer's input
- * scale.  The word is cleared by the read. */
+ * PP_PRECISION_F16X3 an input was not finite or overflowed fp16 (|x s_x| >=
+ * 65520) after the layer's input scale.  The word is cleared by the read. */
 pp_status pp_layer_device_status(const pp_layer* layer, int* device_error);
 
 /* Polls of an mbarrier after which a wait in the tensor-core kernels gives up:

@@ -41,8 +41,9 @@
 // kind::f16), w_hi x_hi into one accumulator and w_lo x_hi + w_hi x_lo into a
 // second one (pixel-major: the lo half of the merged operand's columns and the
 // x_lo MMA; filter-major: the row segment's second TW columns), combined in the
-// epilogue as (acc1 + 2^-11 acc2) times the filter's inverse scale; inputs at
-// or beyond 2^15 after scaling are flagged in the device status word.
+// epilogue as (acc1 + 2^-11 acc2) times the filter's inverse scale; inputs that
+// overflow fp16 after scaling (or are not finite) are flagged in the device
+// status word.
 // Epilogue: bias, +skip, ReLU, 2x2 max pool from tcgen05.ld, stores to each
 // filter's original channel.  This kernel has no channel split: layers with
 // more than 64 filters on maps at most 128 wide can also run the flat kernel
@@ -141,14 +142,18 @@ struct Geo {
   static constexpr int LO_BYTES = IN_BYTES > RAW ? IN_BYTES : RAW;
   static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo (FB x 8 fp32 or FB x 16 f16)
   static constexpr int W_BYTES = NTAP * 2 * W_TILE;       // weights of one chunk
-  // SEP: the raw boxes get a ring of their own (two slots), so the copy for a
-  // chunk can start two chunks ahead instead of waiting for the MMAs that read
-  // the stage; used whenever it fits in shared memory.
+  // SEP: the raw boxes get a ring of their own (NRAW = two slots, or one when
+  // two do not fit), so the copy for chunk g + NRAW starts as soon as chunk g's
+  // box has been read instead of waiting for the MMAs that read the stage; used
+  // whenever it fits in shared memory.  The two raw_full barriers alternate
+  // between chunks whatever the slot count.
   static constexpr int STAGE_SEP = W_BYTES + 2 * IN_BYTES;
-  static constexpr bool SEP = 2 * STAGE_SEP + 2 * RAW + 1024 <= 232448;
+  static constexpr int NRAW = 2 * STAGE_SEP + 2 * RAW + 1024 <= 232448 ? 2
+                              : (2 * STAGE_SEP + RAW + 1024 <= 232448 ? 1 : 0);
+  static constexpr bool SEP = NRAW > 0;
   static constexpr int STAGE = SEP ? STAGE_SEP : W_BYTES + IN_BYTES + LO_BYTES;
   static constexpr int RAW_OFF = 2 * STAGE;               // raw slots (SEP)
-  static constexpr int SMEM_ALLOC = 2 * STAGE + (SEP ? 2 * RAW : 0) + 1024;
+  static constexpr int SMEM_ALLOC = 2 * STAGE + NRAW * RAW + 1024;
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
   static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
   static_assert(W_BYTES % 128 == 0 && IN_BYTES % 128 == 0 && RAW % 128 == 0 && STAGE % 128 == 0,
@@ -262,10 +267,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && G::SEP)
-      for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + G::RAW_OFF + raw_issued * G::RAW);
+      for (; raw_issued < G::NRAW && raw_issued < nall; ++raw_issued)
+        issue_raw(raw_issued, smem + G::RAW_OFF + raw_issued * G::RAW);
     int g = 0;  // chunk sequence number of this CTA
     bool stop = false;  // identical in every loader thread (decided by loader_any)
-    bool range_bad = false;  // f16: an input at or beyond 2^15 after scaling
+    uint32_t range_bad = 0;  // f16: nonzero once an input is non-finite or overflows fp16 after scaling
     for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, (int)blockIdx.x + i * (int)gridDim.x, G::R, TW);
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
@@ -294,12 +300,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             stop = true;
             break;
           }
-          const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g & 1) * G::RAW)
+          const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % G::NRAW) * G::RAW)
                                     : reinterpret_cast<const float*>(lo);
           if constexpr (F16 && G::SEP) {
-            // the box has a slot of its own: each item is split and stored as soon as it is read (fewer
-            // live registers than reading the whole box first); the slot is released after the last read
-#pragma unroll
+            // the box has a slot of its own: each item is split and stored as soon as it is read, one item
+            // per loop trip (few live registers and little code: the f16 split costs several instructions
+            // per value); the slot is released after the last read
+#pragma unroll 1
             for (int b = 0; b < G::ITEMS; ++b) {
               const int it = b * NLOAD + tid;
               if (it < 2 * G::NPIX) {
@@ -318,8 +325,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             group_sync<NLOAD>();
-            if (tid == 0 && raw_issued < nall && raw_issued == g + 2) {
-              issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued & 1) * G::RAW);
+            if (tid == 0 && raw_issued < nall && raw_issued == g + G::NRAW) {
+              issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % G::NRAW) * G::RAW);
               ++raw_issued;
             }
           } else {
@@ -339,8 +346,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           // copy with a proxy fence, then the loader barrier lets thread 0 issue it.
           if (G::SEP) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           group_sync<NLOAD>();  // every raw value is in registers before its slot is reused
-          if (G::SEP && tid == 0 && raw_issued < nall && raw_issued == g + 2) {
-            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued & 1) * G::RAW);
+          if (G::SEP && tid == 0 && raw_issued < nall && raw_issued == g + G::NRAW) {
+            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % G::NRAW) * G::RAW);
             ++raw_issued;
           }
 #pragma unroll
@@ -368,10 +375,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         } else {
           // Items in batches of LBATCH per thread: all global loads of a batch
           // are issued before any is used, so their latencies overlap.
-          for (int base = 0; base < 2 * G::NPIX; base += NLOAD * LBATCH) {
-            float v[LBATCH][G::CPH];
+          constexpr int LB = F16 ? LBATCH / 2 : LBATCH;  // f16 items carry 8 values: the same loads in flight
+          for (int base = 0; base < 2 * G::NPIX; base += NLOAD * LB) {
+            float v[LB][G::CPH];
 #pragma unroll
-            for (int b = 0; b < LBATCH; ++b) {
+            for (int b = 0; b < LB; ++b) {
               const int it = base + b * NLOAD + tid;
               const int kh = it >= G::NPIX ? 1 : 0;
               const int pix = it - kh * G::NPIX;
@@ -385,7 +393,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               }
             }
 #pragma unroll
-            for (int b = 0; b < LBATCH; ++b) {
+            for (int b = 0; b < LB; ++b) {
               const int it = base + b * NLOAD + tid;
               if (it < 2 * G::NPIX) {
                 const int dst = it + (it >= G::NPIX ? G::NPIXA - G::NPIX : 0);
@@ -411,7 +419,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         mbar_arrive(su32(&full[s]));
       }
     }
-    if (F16 && range_bad) atomicOr(p.status, ppc::kStatusF16Range);
+    if (F16 && range_bad != 0) atomicOr(p.status, ppc::kStatusF16Range);
     if (tid == 0) {
       // No copy may still be writing shared memory when the CTA exits: after an
       // early stop, wait (bounded) for the last copies of each kind to land.
@@ -863,8 +871,8 @@ pp_status tc_build(TcLayout* T, const pp_packed* pk, cudaStream_t stream) {
 // 16 + (k % 8) * 2, rows 0 .. FB-1 hi = f16(w s) and FB .. 2 FB-1 lo = f16((w s -
 // hi) * 2^11), with s the filter's scale: the power of two that puts its largest
 // kept |w| in [2^13, 2^14).  The input is scaled by xs, the largest power of two
-// with input_bound * xs <= 2^14, so inputs up to twice the bound stay below 2^15
-// (fp16 holds up to 65504).  rscale[j] = 1 / (s_j xs) for reordered filter j
+// with input_bound * xs <= 2^14, so inputs up to four times the bound stay below
+// 65504, the largest fp16 value.  rscale[j] = 1 / (s_j xs) for reordered filter j
 // (1 / xs for an empty filter and past Co).  Conversions round to nearest.
 pp_status tc_build16(TcLayout* T, const pp_packed* pk, float input_bound, cudaStream_t stream) {
   const int Co = pk->Co, Ci = pk->Ci, FB = T->FB;

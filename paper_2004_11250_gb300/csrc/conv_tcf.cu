@@ -34,8 +34,9 @@
 // accumulator and w_lo x_hi + w_hi x_lo into a second one (TMEM columns 128 ..
 // 255 of the buffer), combined in the epilogue as (acc1 + 2^-11 acc2) times the
 // filter's inverse scale.  The dropped lo x lo term and the rounding of the lo
-// parts are each below 2^-22 of |w * x|.  Inputs at or beyond 2^15 after
-// scaling would overflow fp16: the loaders flag them in the device status word.
+// parts are each below 2^-22 of |w * x|.  Inputs that overflow fp16 after
+// scaling (|x s| >= 65520) or are not finite are flagged by the loaders in the
+// device status word.
 //
 // Roles (17 warps, one CTA per SM): warps 0-7 stage the operands, warp 8
 // allocates TMEM and one of its threads issues the MMAs, warps 9-16 are the
@@ -96,7 +97,7 @@ struct FlatParams {
   int nch, nfb, flags, use_tma;
   int bcols, R, ncols, npix, npixa, raw_w, raw_bytes;
   int stage, lo_off;        // bytes per stage; offset of the lo operand in a stage (hi is at W_BYTES)
-  int sep, raw_off, raw_slot;  // input boxes in a ring of their own (two slots at raw_off)
+  int sep, raw_off, raw_slot;  // input boxes in a ring of their own: sep (2 or 1) slots at raw_off; 0 = none
   int tiles_y, ntiles, split;
   uint32_t idesc;
 };
@@ -311,8 +312,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           "r"(su32(&raw_full[gg & 1]))
           : "memory");
     };
-    // With a ring of their own the boxes are copied two chunks ahead of use,
-    // not only once the chunk's stage is free.
+    // With a ring of their own the boxes are copied one or two chunks ahead of use
+    // (as many as the ring has slots), not only once the chunk's stage is free.
     // Weights of chunk gg into stage s (thread 0).
     auto issue_w = [&](int gg, int s) {
       const Tile T = tile_of(p, tile_index(gg / nchm));
@@ -332,9 +333,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && p.sep)
-      for (; raw_issued < 2 && raw_issued < nall; ++raw_issued) issue_raw(raw_issued, smem + p.raw_off + raw_issued * p.raw_slot);
+      for (; raw_issued < p.sep && raw_issued < nall; ++raw_issued)
+        issue_raw(raw_issued, smem + p.raw_off + raw_issued * p.raw_slot);
     bool stop = false;  // identical in every loader thread (decided by group_any)
-    bool range_bad = false;  // f16: an input at or beyond 2^15 after scaling
+    uint32_t range_bad = 0;  // f16: nonzero once an input is non-finite or overflows fp16 after scaling
     for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, tile_index(i));
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
@@ -378,7 +380,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             stop = true;
             break;
           }
-          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)s * p.raw_slot)
+          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g % p.sep) * p.raw_slot)
                                    : reinterpret_cast<const float*>(lo);
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b)
@@ -388,8 +390,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           // thread orders its reads of the slot before that copy with a proxy fence.
           if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           group_sync<NLOAD>();  // the whole box is in registers before its buffer is reused
-          if (p.sep && tid == 0 && raw_issued < nall && raw_issued == g + 2) {
-            issue_raw(raw_issued, smem + p.raw_off + (size_t)s * p.raw_slot);
+          if (p.sep && tid == 0 && raw_issued < nall && raw_issued == g + p.sep) {
+            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued % p.sep) * p.raw_slot);
             ++raw_issued;
           }
         }
@@ -417,7 +419,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         mbar_arrive(su32(&full[s]));
       }
     }
-    if (F16 && range_bad) atomicOr(p.status, ppc::kStatusF16Range);
+    if (F16 && range_bad != 0) atomicOr(p.status, ppc::kStatusF16Range);
     if (tid == 0) {
       // No copy may still be writing shared memory when the CTA exits: wait
       // (bounded) for the last copies issued into each stage.
@@ -780,7 +782,8 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
     const int in_bytes = (2 * G.npixa * 16 + 127) / 128 * 128;
     G.raw_slot = (G.raw_bytes + 127) / 128 * 128;
     G.stage = W_BYTES + 2 * in_bytes;
-    G.sep = 2 * G.stage + 2 * G.raw_slot <= SMEM_USE;
+    // a ring of two box slots, else one (copied one chunk ahead), else the box lands in the stage
+    G.sep = 2 * G.stage + 2 * G.raw_slot <= SMEM_USE ? 2 : (2 * G.stage + G.raw_slot <= SMEM_USE ? 1 : 0);
     if (!G.sep) G.stage = W_BYTES + in_bytes + std::max(in_bytes, G.raw_slot);  // the box lands in lo
     G.lo_off = W_BYTES + in_bytes;
     G.raw_off = 2 * G.stage;

@@ -103,20 +103,22 @@ __device__ __forceinline__ float tf32_hi(float v) { return __uint_as_float(__flo
 // fp16 split of 8 fp32 values scaled by sc (a power of two): hi = f16(v sc) and
 // lo = f16((v sc - hi) * 2^11), rounded to nearest, 8 halves per 16 bytes in the
 // values' order (the K-major row of a kind::f16 operand).  v sc - hi is exact in
-// fp32.  Returns true when a scaled value is at or beyond 2^15 (fp16 overflow
-// territory); NaN is not flagged (it propagates as in fp32).
-__device__ __forceinline__ bool split_f16x8(const float* v, float sc, uint4& h, uint4& l) {
+// fp32.  Returns a word that is nonzero when some hi half is infinite or NaN,
+// i.e. |v sc| >= 65520 (fp16 overflow) or v is not a number: for every half the
+// exponent field plus one carries into the cleared sign bit exactly when it is
+// all ones.
+__device__ __forceinline__ uint32_t split_f16x8(const float* v, float sc, uint4& h, uint4& l) {
   uint32_t hw[4], lw[4];
-  bool bad = false;
+  uint32_t bad = 0;
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     const float a = v[2 * k] * sc, b = v[2 * k + 1] * sc;
-    bad |= fabsf(a) >= 32768.f || fabsf(b) >= 32768.f;
     const __half2 hh = __floats2half2_rn(a, b);
     const float2 hf = __half22float2(hh);
     const __half2 ll = __floats2half2_rn((a - hf.x) * 2048.f, (b - hf.y) * 2048.f);
     hw[k] = *reinterpret_cast<const uint32_t*>(&hh);
     lw[k] = *reinterpret_cast<const uint32_t*>(&ll);
+    bad |= ((hw[k] & 0x7FFF7FFFu) + 0x04000400u) & 0x80008000u;
   }
   h = make_uint4(hw[0], hw[1], hw[2], hw[3]);
   l = make_uint4(lw[0], lw[1], lw[2], lw[3]);

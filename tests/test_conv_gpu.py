@@ -874,14 +874,14 @@ def test_f16_sweep_point(pp, runner, oracle_mod, point):
 
 @pytest.mark.parametrize("kernel", ["TC", "TC_FLAT"])
 def test_f16_input_range(pp, runner, oracle_mod, kernel):
-    """An input at 2^15 or beyond (after the layer's input scale) is flagged in the device status word
-    (bit 1), not silently wrong; with a bound that covers it (input scale 2^-3 for a bound of 1e5) the
-    same input is within the error bound; the precision and scale read back."""
+    """An input that overflows fp16 after the layer's input scale (70000 at scale 1) is flagged in the
+    device status word (bit 1), not silently wrong; with a bound that covers it (input scale 2^-3 for a
+    bound of 1e5) the same input is within the error bound; the precision and scale read back."""
     rng = np.random.default_rng(5)
     Co, Ci, N, H, W = 136, 16, 1, 12, 20
     L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.5)
     x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
-    x[0, 3, 5, 7] = 40000.0
+    x[0, 3, 5, 7] = 70000.0
     dl = runner.DeviceLayer(L, precision=F16)
     try:
         pp.pp_layer_set_kernel(dl.handle, getattr(pp, "PP_KERNEL_" + kernel))
