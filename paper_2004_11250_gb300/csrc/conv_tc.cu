@@ -80,6 +80,8 @@ constexpr int NEPI = 256;          // epilogue threads
 constexpr int NTHREADS = 544;
 constexpr int LBATCH = 4;          // loader items whose global loads are in flight together
 constexpr long WAIT_LIMIT = PP_WAIT_POLLS;  // mbarrier polls before a wait gives up
+// dynamic shared memory a CTA may request: 227 KB less room for the kernel's static barriers
+constexpr int SMEM_LIMIT = 232448 - 256;
 
 // Orientation of the GEMM on the tensor core.
 //   ORI_FP: M = 128 filters, N = TW pixels of one output row (narrow maps)
@@ -148,14 +150,14 @@ struct Geo {
   // whenever it fits in shared memory.  The two raw_full barriers alternate
   // between chunks whatever the slot count.
   static constexpr int STAGE_SEP = W_BYTES + 2 * IN_BYTES;
-  static constexpr int NRAW = 2 * STAGE_SEP + 2 * RAW + 1024 <= 232448 ? 2
-                              : (2 * STAGE_SEP + RAW + 1024 <= 232448 ? 1 : 0);
+  static constexpr int NRAW = 2 * STAGE_SEP + 2 * RAW + 1024 <= SMEM_LIMIT ? 2
+                              : (2 * STAGE_SEP + RAW + 1024 <= SMEM_LIMIT ? 1 : 0);
   static constexpr bool SEP = NRAW > 0;
   static constexpr int STAGE = SEP ? STAGE_SEP : W_BYTES + IN_BYTES + LO_BYTES;
   static constexpr int RAW_OFF = 2 * STAGE;               // raw slots (SEP)
   static constexpr int SMEM_ALLOC = 2 * STAGE + NRAW * RAW + 1024;
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
-  static_assert(SMEM_ALLOC <= 232448, "shared memory plan");
+  static_assert(SMEM_ALLOC <= SMEM_LIMIT, "shared memory plan");
   static_assert(W_BYTES % 128 == 0 && IN_BYTES % 128 == 0 && RAW % 128 == 0 && STAGE % 128 == 0,
                 "tensor-map copies need 128-byte aligned shared-memory destinations");
   static constexpr uint32_t IDESC = F16 ? (ORI == ORI_FP ? idesc_f16(128, TW) : idesc_f16(128, FB))
