@@ -328,6 +328,33 @@ def time_ops_in_frame(dn, acts, steps, flush, stream):
     return [statistics.median(v) for v in per]
 
 
+def time_graph_of_launches(dn, acts, reps, steps, stream):
+    """Per-launch time (ms) of op 0 replayed back to back: one CUDA graph of `reps` launches of the op on the
+    same buffers (no L2 flush between them: weights and input stay warm), replayed `steps` times.  With a
+    launch far shorter than the launch latency this separates the kernel's own time from the latency of a
+    lone launch."""
+    import torch
+    from paper_2004_11250_gb300 import runner
+    op, L = dn.spec.ops[0], dn.layers[0]
+    xin, out = acts[0], acts[1]
+    N, _, H, W = xin.shape
+    flags = runner.op_flags(op)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for _ in range(reps):
+            L.forward(xin, out, None, N, H, W, flags, torch.cuda.current_stream())
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        g.replay()
+    e1.record(stream)
+    e1.synchronize()
+    return e0.elapsed_time(e1) / (steps * reps)
+
+
 def traffic_from_profile(kernel_hash: str, kernel: str = None):
     """Per-launch DRAM bytes (read + write) from the committed ncu summary of the VGG-16 frame, of one
     kernel (average over its launches in the frame) or of all the frame's convs, if that summary was
@@ -401,11 +428,18 @@ def bench_config(name, steps, warmup, flush, stream, hbm, fold_too=False, precis
         per_op = [KERNEL_NAMES.get(pp.pp_layer_kernel(L.handle), "?") if not L.dense else "dense" for L in dn.layers]
         kern = sorted(set(k for k in per_op if k != "dense"))
         tv = tensor_view(shapes, per_op, op_ms, [k for k, s in enumerate(shapes) if s["pruned"]], f16=precision == 1)
+        graph_us = None
+        if name == "single":
+            graph_us = round(time_graph_of_launches(dn, dn.run_layerwise(x), 20, 10, stream) * 1e3, 3)
         res = {"ms_per_frame": round(ms, 4), "gflops": round(flops / (ms * 1e-3) / 1e9, 1), "kernels": kern,
                "op_us_in_frame": [round(t * 1e3, 2) for t in op_ms],
                "roofline_frac_min_pruned_op": round(min(pr), 3) if pr else None,
                "roofline_frac_median_pruned_op": round(statistics.median(pr), 3) if pr else None,
                "tensor_tflops": tv["achieved"] if tv else None, "tensor_frac": tv["frac"] if tv else None}
+        if graph_us is not None:
+            res["us_per_launch_graph_of_20"] = graph_us
+            res["roofline_frac_graph_of_20"] = round(roof_time_s(shapes[0]["flops"], shapes[0]["bytes"], hbm)
+                                                     / (graph_us * 1e-6), 4)
     finally:
         dn.close()
     if fold_too:
@@ -719,6 +753,7 @@ def main():
             "gpu_launches": len(spec.ops) * args.steps,
             "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
                          "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
+                         "frac_of_derived_peak": round(achieved / peaks["derived_fp32_tflops"], 4),
                          "kernel": f"{dom} ({len(dom_ops)} of the {len(pruned)} pruned convs, "
                                    f"{100 * by_kern[dom][1] / kt:.0f}% of their in-frame device time)",
                          "timing": "op by op in frame order, CUDA events between the ops on the launching "
