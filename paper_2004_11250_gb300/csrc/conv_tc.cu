@@ -279,6 +279,39 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
       for (int c = 0; c < p.nch; ++c, ++g) {
         const int s = g & 1, use = g >> 1;
+        // f16 with a box ring: the box of this chunk has a slot of its own and lands ahead of time, so it is
+        // read and split into registers before the stage is free (while the MMAs of the two previous chunks
+        // still read it); only the stores wait for the stage.
+        constexpr int EI = (F16 && G::SEP) ? G::ITEMS : 1;
+        uint4 hreg[EI], lreg[EI];
+        const bool early = F16 && G::SEP && p.use_tma;
+        if (early) {
+          if (group_any<NLOAD>(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
+            stop = true;
+            break;
+          }
+          const float* raw = reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % G::NRAW) * G::RAW);
+#pragma unroll
+          for (int b = 0; b < EI; ++b) {
+            const int it = b * NLOAD + tid;
+            if (it < 2 * G::NPIX) {
+              const int kh = it >= G::NPIX ? 1 : 0;
+              const int pix = it - kh * G::NPIX;
+              const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
+              float u[G::CPH];
+#pragma unroll
+              for (int k = 0; k < G::CPH; ++k) u[k] = raw[((kh * G::CPH + k) * G::BROWS + br) * G::RAW_W + bc + 3];
+              range_bad |= split_f16x8(u, p.xscale, hreg[b], lreg[b]);
+            }
+          }
+          // the slot is rewritten next by a tensor-map copy: reads ordered before it, then released
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          group_sync<NLOAD>();
+          if (tid == 0 && raw_issued < nall && raw_issued == g + G::NRAW) {
+            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % G::NRAW) * G::RAW);
+            ++raw_issued;
+          }
+        }
         if (group_any<NLOAD>(use > 0 && !wait(&empty[s], (uint32_t)((use - 1) & 1)))) {
           stop = true;
           break;
@@ -297,41 +330,23 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           }
         }
         const int ch0 = c * G::KCH;
-        if (p.use_tma) {
+        if (early) {
+#pragma unroll
+          for (int b = 0; b < EI; ++b) {
+            const int it = b * NLOAD + tid;
+            if (it < 2 * G::NPIX) {
+              const int dst = it + (it >= G::NPIX ? G::NPIXA - G::NPIX : 0);  // K halves NPIXA apart
+              reinterpret_cast<uint4*>(hi)[dst] = hreg[b];
+              reinterpret_cast<uint4*>(lo)[dst] = lreg[b];
+            }
+          }
+        } else if (p.use_tma) {
           if (group_any<NLOAD>(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
             stop = true;
             break;
           }
           const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % G::NRAW) * G::RAW)
                                     : reinterpret_cast<const float*>(lo);
-          if constexpr (F16 && G::SEP) {
-            // the box has a slot of its own: each item is split and stored as soon as it is read, one item
-            // per loop trip (few live registers and little code: the f16 split costs several instructions
-            // per value); the slot is released after the last read
-#pragma unroll 1
-            for (int b = 0; b < G::ITEMS; ++b) {
-              const int it = b * NLOAD + tid;
-              if (it < 2 * G::NPIX) {
-                const int kh = it >= G::NPIX ? 1 : 0;
-                const int pix = it - kh * G::NPIX;
-                const int br = pix / G::BCOLS, bc = pix - br * G::BCOLS;
-                float u[G::CPH];
-#pragma unroll
-                for (int k = 0; k < G::CPH; ++k) u[k] = raw[((kh * G::CPH + k) * G::BROWS + br) * G::RAW_W + bc + 3];
-                uint4 h, l;
-                range_bad |= split_f16x8(u, p.xscale, h, l);
-                const int dst = it + (kh ? G::NPIXA - G::NPIX : 0);  // K halves NPIXA apart
-                reinterpret_cast<uint4*>(hi)[dst] = h;
-                reinterpret_cast<uint4*>(lo)[dst] = l;
-              }
-            }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            group_sync<NLOAD>();
-            if (tid == 0 && raw_issued < nall && raw_issued == g + G::NRAW) {
-              issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % G::NRAW) * G::RAW);
-              ++raw_issued;
-            }
-          } else {
           float v[G::ITEMS][G::CPH];
 #pragma unroll
           for (int b = 0; b < G::ITEMS; ++b) {
@@ -372,7 +387,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
                 lo[dst] = make_float4(v[b][0] - h.x, v[b][1] - h.y, v[b][2] - h.z, v[b][3] - h.w);
               }
             }
-          }
           }
         } else {
           // Items in batches of LBATCH per thread: all global loads of a batch

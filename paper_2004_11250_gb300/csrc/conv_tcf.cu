@@ -344,7 +344,49 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         const int s = g & 1, use = g >> 1;
         // Without a tensor map the chunk's input values are fetched into
         // registers first: that needs no free stage, so it overlaps the wait.
+        // With a box ring the box has a slot of its own and lands ahead of time:
+        // it is read (and, for f16, split) into registers before the stage is
+        // free too, while the MMAs of the two previous chunks still read it.
+        // v holds an item's input values, or (f16, split early) its packed hi words then lo words
         float v[ITEMS_MAX][CPH];
+        const bool early = p.use_tma && p.sep;
+        if (early) {
+          if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
+            stop = true;
+            break;
+          }
+          const float* raw = reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g % p.sep) * p.raw_slot);
+#pragma unroll
+          for (int b = 0; b < ITEMS_MAX; ++b) {
+            if constexpr (F16) {
+              // split as soon as read: only the packed halves stay live
+              float u[CPH];
+#pragma unroll
+              for (int k = 0; k < CPH; ++k) u[k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+              uint4 h = make_uint4(0, 0, 0, 0), l = h;
+              if (doff[b] >= 0) range_bad |= split_f16x8(u, p.xscale, h, l);
+              v[b][0] = __uint_as_float(h.x);
+              v[b][1] = __uint_as_float(h.y);
+              v[b][2] = __uint_as_float(h.z);
+              v[b][3] = __uint_as_float(h.w);
+              v[b][4] = __uint_as_float(l.x);
+              v[b][5] = __uint_as_float(l.y);
+              v[b][6] = __uint_as_float(l.z);
+              v[b][7] = __uint_as_float(l.w);
+            } else {
+#pragma unroll
+              for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+            }
+          }
+          // the slot is rewritten next by a tensor-map copy (async proxy): each thread orders its reads of
+          // it before that copy with a proxy fence, then the loader barrier lets thread 0 issue it
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          group_sync<NLOAD>();
+          if (tid == 0 && raw_issued < nall && raw_issued == g + p.sep) {
+            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued % p.sep) * p.raw_slot);
+            ++raw_issued;
+          }
+        }
         if (!p.use_tma) {
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b) {
@@ -375,25 +417,18 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             ++raw_issued;
           }
         }
-        if (p.use_tma) {
+        if (p.use_tma && !early) {
+          // no ring: the box landed in the lo operand of this stage
           if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
             stop = true;
             break;
           }
-          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g % p.sep) * p.raw_slot)
-                                   : reinterpret_cast<const float*>(lo);
+          const float* raw = reinterpret_cast<const float*>(lo);
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b)
 #pragma unroll
             for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
-          // A ring slot is rewritten next by a tensor-map copy (async proxy): each
-          // thread orders its reads of the slot before that copy with a proxy fence.
-          if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          group_sync<NLOAD>();  // the whole box is in registers before its buffer is reused
-          if (p.sep && tid == 0 && raw_issued < nall && raw_issued == g + p.sep) {
-            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued % p.sep) * p.raw_slot);
-            ++raw_issued;
-          }
+          group_sync<NLOAD>();  // the whole box is in registers before the lo operand is written over it
         }
 #pragma unroll
         for (int b = 0; b < ITEMS_MAX; ++b) {
@@ -401,7 +436,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             const int dst = doff[b];
             if constexpr (F16) {
               uint4 h, l;
-              range_bad |= split_f16x8(&v[b][0], p.xscale, h, l);
+              if (early) {
+                h = make_uint4(__float_as_uint(v[b][0]), __float_as_uint(v[b][1]), __float_as_uint(v[b][2]),
+                               __float_as_uint(v[b][3]));
+                l = make_uint4(__float_as_uint(v[b][4]), __float_as_uint(v[b][5]), __float_as_uint(v[b][6]),
+                               __float_as_uint(v[b][7]));
+              } else {
+                range_bad |= split_f16x8(&v[b][0], p.xscale, h, l);
+              }
               reinterpret_cast<uint4*>(hi)[dst] = h;
               reinterpret_cast<uint4*>(lo)[dst] = l;
             } else {
