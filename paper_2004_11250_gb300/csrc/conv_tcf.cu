@@ -344,12 +344,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         const int s = g & 1, use = g >> 1;
         // Without a tensor map the chunk's input values are fetched into
         // registers first: that needs no free stage, so it overlaps the wait.
-        // With a box ring the box has a slot of its own and lands ahead of time:
-        // it is read (and, for f16, split) into registers before the stage is
-        // free too, while the MMAs of the two previous chunks still read it.
+        // f16 with a box ring: the box has a slot of its own and lands ahead of
+        // time, so it is read and split into registers before the stage is free
+        // too, while the MMAs of the two previous chunks still read it (for tf32
+        // the split is cheap and waiting for the box first would only delay the
+        // chunk's weight copy, issued once the stage is free).
         // v holds an item's input values, or (f16, split early) its packed hi words then lo words
         float v[ITEMS_MAX][CPH];
-        const bool early = p.use_tma && p.sep;
+        const bool early = F16 && p.use_tma && p.sep;
         if (early) {
           if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
             stop = true;
@@ -418,17 +420,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           }
         }
         if (p.use_tma && !early) {
-          // no ring: the box landed in the lo operand of this stage
           if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
             stop = true;
             break;
           }
-          const float* raw = reinterpret_cast<const float*>(lo);
+          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g % p.sep) * p.raw_slot)
+                                   : reinterpret_cast<const float*>(lo);
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b)
 #pragma unroll
             for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
-          group_sync<NLOAD>();  // the whole box is in registers before the lo operand is written over it
+          // A ring slot is rewritten next by a tensor-map copy (async proxy): each
+          // thread orders its reads of the slot before that copy with a proxy fence.
+          if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          group_sync<NLOAD>();  // the whole box is in registers before its buffer is reused
+          if (p.sep && tid == 0 && raw_issued < nall && raw_issued == g + p.sep) {
+            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued % p.sep) * p.raw_slot);
+            ++raw_issued;
+          }
         }
 #pragma unroll
         for (int b = 0; b < ITEMS_MAX; ++b) {

@@ -53,15 +53,8 @@ __global__ void __launch_bounds__(FFMA_THREADS) ffma_probe_kernel(long long iter
     ns0 = globaltimer();
     clk0 = clock64();
   }
-  // 8 rounds of the chains per loop trip, so the loop's own instructions take few issue slots
-  long long i = 0;
-  for (; i + 8 <= iters; i += 8) {
-#pragma unroll
-    for (int r = 0; r < 8; ++r)
-#pragma unroll
-      for (int k = 0; k < FFMA_CHAINS; ++k) a[k] = fmaf(a[k], b, c);
-  }
-  for (; i < iters; ++i) {
+  // (a loop unrolled 8 rounds deep measured ~4 % lower on GB300 than this one)
+  for (long long i = 0; i < iters; ++i) {
 #pragma unroll
     for (int k = 0; k < FFMA_CHAINS; ++k) a[k] = fmaf(a[k], b, c);
   }
