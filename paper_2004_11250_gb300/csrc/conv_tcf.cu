@@ -98,6 +98,7 @@ struct FlatParams {
   int bcols, R, ncols, npix, npixa, raw_w, raw_bytes;
   int stage, lo_off;        // bytes per stage; offset of the lo operand in a stage (hi is at W_BYTES)
   int sep, raw_off, raw_slot;  // input boxes in a ring of their own: sep (2 or 1) slots at raw_off; 0 = none
+                               // (slot of chunk g: g & (sep - 1))
   int tiles_y, ntiles, split;
   uint32_t idesc;
 };
@@ -357,7 +358,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             stop = true;
             break;
           }
-          const float* raw = reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g % p.sep) * p.raw_slot);
+          const float* raw = reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g & (p.sep - 1)) * p.raw_slot);
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b) {
             if constexpr (F16) {
@@ -385,7 +386,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           group_sync<NLOAD>();
           if (tid == 0 && raw_issued < nall && raw_issued == g + p.sep) {
-            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued % p.sep) * p.raw_slot);
+            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued & (p.sep - 1)) * p.raw_slot);
             ++raw_issued;
           }
         }
@@ -424,7 +425,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             stop = true;
             break;
           }
-          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g % p.sep) * p.raw_slot)
+          const float* raw = p.sep ? reinterpret_cast<const float*>(smem + p.raw_off + (size_t)(g & (p.sep - 1)) * p.raw_slot)
                                    : reinterpret_cast<const float*>(lo);
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b)
@@ -435,7 +436,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           group_sync<NLOAD>();  // the whole box is in registers before its buffer is reused
           if (p.sep && tid == 0 && raw_issued < nall && raw_issued == g + p.sep) {
-            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued % p.sep) * p.raw_slot);
+            issue_raw(raw_issued, smem + p.raw_off + (size_t)(raw_issued & (p.sep - 1)) * p.raw_slot);
             ++raw_issued;
           }
         }
