@@ -738,24 +738,28 @@ extern "C" pp_status pp_layer_set_output_order(pp_layer* L, const int32_t* order
     seen[ord[o]] = 1;
   }
   cudaStream_t stream = (cudaStream_t)stream_;
-  // every kernel but the direct one stores reordered filter j at channel perm[j]
-  std::vector<int32_t> store(Co);
-  for (int j = 0; j < Co; ++j) store[j] = ord[L->pk_perm[j]];
-  if (cudaMemcpyAsync(L->perm, store.data(), (size_t)Co * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
-      cudaStreamSynchronize(stream) != cudaSuccess) {
-    cudaGetLastError();
-    return PP_ERR_CUDA;
-  }
+  // the direct kernel stores row o of its dense weights at channel o: its layout is rebuilt with rows
+  // moved, first, so that a failure leaves the layer as it was
+  ppc::DirectLayout D;
   if (L->direct.w) {
-    // the direct kernel stores row o of its dense weights at channel o: rebuild them with rows moved
     std::vector<float> w((size_t)Co * Ci * 9), b(L->direct_bias.empty() ? 0 : Co);
     for (int o = 0; o < Co; ++o) {
       std::memcpy(&w[(size_t)ord[o] * Ci * 9], &L->direct_w[(size_t)o * Ci * 9], (size_t)Ci * 9 * sizeof(float));
       if (!b.empty()) b[ord[o]] = L->direct_bias[o];
     }
-    ppc::DirectLayout D;
     const pp_status st = ppc::direct_build(&D, w.data(), b.empty() ? nullptr : b.data(), Co, Ci, stream);
     if (st != PP_OK) return st;
+  }
+  // every other kernel stores reordered filter j at channel perm[j]
+  std::vector<int32_t> store(Co);
+  for (int j = 0; j < Co; ++j) store[j] = ord[L->pk_perm[j]];
+  if (cudaMemcpyAsync(L->perm, store.data(), (size_t)Co * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess) {
+    cudaGetLastError();
+    ppc::direct_free(&D);
+    return PP_ERR_CUDA;
+  }
+  if (L->direct.w) {
     ppc::direct_free(&L->direct);
     L->direct = D;
   }
