@@ -686,7 +686,9 @@ extern "C" pp_status pp_layer_create(const pp_packed* pk, const float* bias, voi
     if (st == PP_OK) st = ppc::tm_build(&L->tm, pk, rmap, (cudaStream_t)stream);
     L->tm_ok = st == PP_OK;
   }
-  if (st == PP_OK && pk->Ci >= 8) {
+  if (st == PP_OK) {
+    // channels are padded to the chunk width (zero weights, zero-filled input
+    // boxes), so a layer with fewer than 8 input channels has one ragged chunk
     st = ppc::tc_prepare();
     if (st == PP_OK) st = ppc::tc_build(&L->tc, pk, (cudaStream_t)stream);
     L->tc_ok = st == PP_OK;

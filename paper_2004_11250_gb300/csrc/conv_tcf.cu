@@ -99,6 +99,7 @@ struct FlatParams {
   int stage, lo_off;        // bytes per stage; offset of the lo operand in a stage (hi is at W_BYTES)
   int sep, raw_off, raw_slot;  // input boxes in a ring of their own: sep (2 or 1) slots at raw_off; 0 = none
                                // (slot of chunk g: g & (sep - 1))
+  int plane;                // box over x viewed as [N][Ci][H * W]: the staged rows packed, raw_w = box width
   int tiles_y, ntiles, split;
   uint32_t idesc;
 };
@@ -295,17 +296,36 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       const int pix = it - kh * p.npix;
       const int br = pix / p.bcols, bc = pix - br * p.bcols;
       const bool has = it < 2 * p.npix;
-      roff[b] = has ? (kh * CPH * brows + br) * p.raw_w + bc + 3 : -1;
+      // 4-D box: columns from -4, zero filled outside the image.  Packed rows
+      // (plane): row br of the tile starts br * W elements into the box (after
+      // the tile's alignment shift, added per tile); the halo columns, which
+      // the packed rows do not hold, are zeros.
+      roff[b] = !has ? -1
+                     : (p.plane ? ((bc >= 1 && bc <= p.W) ? kh * CPH * p.raw_w + br * p.W + bc - 1 : -1)
+                                : (kh * CPH * brows + br) * p.raw_w + bc + 3);
       doff[b] = has ? kh * p.npixa + pix : -1;
       rowcol[b] = (kh << 30) | (br << 15) | bc;
     }
-    const int cstride = brows * p.raw_w;  // between two channels of the box
+    const int cstride = p.plane ? p.raw_w : brows * p.raw_w;  // between two channels of the box
+    // Packed rows: the box starts at element (r0 - 1) W rounded down to a
+    // multiple of 4 (16 bytes, as a tensor-map copy requires); the remainder is
+    // the tile's shift into the box.
+    auto plane_shift = [&](const Tile& T) -> int { return p.plane ? ((T.r0 - 1) * p.W) & 3 : 0; };
     // Input box of chunk gg (thread 0): [8 channels][rows r0-1 ..][columns -4 ..];
     // zero fill outside the image is the convolution's padding.
     auto issue_raw = [&](int gg, unsigned char* dst) {
       const int i = gg / nchm, c = c_beg + gg % nchm;
       const Tile T = tile_of(p, tile_index(i));
       mbar_arrive_expect_tx(su32(&raw_full[gg & 1]), (uint32_t)p.raw_bytes);
+      if (p.plane) {
+        const int x0 = (T.r0 - 1) * p.W - plane_shift(T);
+        asm volatile(
+            "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+            "%4}], [%5];" ::"r"(su32(dst)),
+            "l"(reinterpret_cast<uint64_t>(&xmap)), "r"(x0), "r"(c * KCH), "r"(T.n), "r"(su32(&raw_full[gg & 1]))
+            : "memory");
+        return;
+      }
       asm volatile(
           "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
           "%4, %5}], [%6];" ::"r"(su32(dst)),
@@ -341,6 +361,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     for (int i = 0; i < nmine && !stop; ++i) {
       const Tile T = tile_of(p, tile_index(i));
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
+      const int tsh = plane_shift(T);
       for (int c = c_beg; c < c_end; ++c, ++g) {
         const int s = g & 1, use = g >> 1;
         // Without a tensor map the chunk's input values are fetched into
@@ -365,7 +386,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
               // split as soon as read: only the packed halves stay live
               float u[CPH];
 #pragma unroll
-              for (int k = 0; k < CPH; ++k) u[k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+              for (int k = 0; k < CPH; ++k) u[k] = roff[b] >= 0 ? raw[roff[b] + tsh + k * cstride] : 0.f;
               uint4 h = make_uint4(0, 0, 0, 0), l = h;
               if (doff[b] >= 0) range_bad |= split_f16x8(u, p.xscale, h, l);
               v[b][0] = __uint_as_float(h.x);
@@ -378,7 +399,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
               v[b][7] = __uint_as_float(l.w);
             } else {
 #pragma unroll
-              for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+              for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + tsh + k * cstride] : 0.f;
             }
           }
           // the slot is rewritten next by a tensor-map copy (async proxy): each thread orders its reads of
@@ -430,7 +451,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
 #pragma unroll
           for (int b = 0; b < ITEMS_MAX; ++b)
 #pragma unroll
-            for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + k * cstride] : 0.f;
+            for (int k = 0; k < CPH; ++k) v[b][k] = roff[b] >= 0 ? raw[roff[b] + tsh + k * cstride] : 0.f;
           // A ring slot is rewritten next by a tensor-map copy (async proxy): each
           // thread orders its reads of the slot before that copy with a proxy fence.
           if (p.sep) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -963,7 +984,9 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   CUtensorMap xmap;
   std::memset(&xmap, 0, sizeof(xmap));
   p.use_tma = 0;
-  if ((W & 3) == 0 && (reinterpret_cast<uintptr_t>(x) & 15) == 0 && D->encode) {
+  p.plane = 0;
+  const bool can_map = (reinterpret_cast<uintptr_t>(x) & 15) == 0 && D->encode;
+  if (can_map && (W & 3) == 0) {
     // 4-D map over x viewed as [N][Ci][H][W] (W innermost), box [1][8][R+2][BCOLS+4]
     const cuuint64_t dims[4] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)M.Ci, (cuuint64_t)N};
     const cuuint64_t strides[3] = {(cuuint64_t)W * 4, (cuuint64_t)W * H * 4, (cuuint64_t)W * H * M.Ci * 4};
@@ -974,6 +997,25 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
                       ? 1
                       : 0;
+  } else if (can_map && ((size_t)H * W) % 4 == 0) {
+    // Rows not 16-byte aligned but planes are: a 3-D map over x viewed as
+    // [N][Ci][H * W] and a box of the tile's R + 2 rows packed, plus up to 3
+    // elements of alignment shift (the halo columns are zeros in the loaders).
+    const int boxw = ((G.R + 2) * W + 3 + 3) / 4 * 4;
+    if (boxw <= 256 && kch * boxw * 4 <= G.raw_slot) {
+      const cuuint64_t dims[3] = {(cuuint64_t)H * W, (cuuint64_t)M.Ci, (cuuint64_t)N};
+      const cuuint64_t strides[2] = {(cuuint64_t)H * W * 4, (cuuint64_t)H * W * M.Ci * 4};
+      const cuuint32_t box[3] = {(cuuint32_t)boxw, (cuuint32_t)kch, 1};
+      const cuuint32_t estr[3] = {1, 1, 1};
+      if (D->encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(x), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
+        p.use_tma = 1;
+        p.plane = 1;
+        p.raw_w = boxw;
+        p.raw_bytes = kch * boxw * 4;
+      }
+    }
   }
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute at[2];

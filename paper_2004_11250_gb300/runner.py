@@ -47,7 +47,7 @@ class DeviceLayer:
         else:
             self.packed = pp.pp_pack_layer(w, mask, layer.taps)
             self.handle = pp.pp_layer_create(self.packed, layer.bias, stream)
-            if precision != pp.PP_PRECISION_TF32X3 and layer.Ci >= 8:  # layers with a tensor-core layout
+            if precision != pp.PP_PRECISION_TF32X3:
                 pp.pp_layer_set_precision(self.handle, precision, input_bound, stream)
 
     def perm(self) -> np.ndarray:

@@ -104,10 +104,10 @@ def test_register_kernel_on_ring_layers(pp, runner, oracle_mod, case, flags):
     check_within(g, y, s, f"register kernel {case} {flags}")
 
 
-@pytest.mark.parametrize("case", [c for c in SMALL if c[1] >= 8])
+@pytest.mark.parametrize("case", SMALL)
 @pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
 def test_tensor_core_kernel(pp, runner, oracle_mod, case, flags):
-    """The 3xTF32 implicit-GEMM kernel on every small case with at least 8 input channels."""
+    """The 3xTF32 implicit-GEMM kernel on every small case (fewer than 8 input channels: one ragged chunk)."""
     N, Ci, Co, H, W, P, ring, keep = case
     if flags == "pool_relu" and (H % 2 or W % 2):
         pytest.skip("pool needs even sizes")
@@ -118,6 +118,28 @@ def test_tensor_core_kernel(pp, runner, oracle_mod, case, flags):
     g = run_layer(pp, runner, L, x, skip, flags != "none", flags == "pool_relu", kernel=pp.PP_KERNEL_TC)
     y, s = oracle_layer_full(oracle_mod, L, x, skip, flags != "none", flags == "pool_relu")
     check_within(g, y, s, f"tensor-core kernel {case} {flags}")
+
+
+@pytest.mark.parametrize("shape,flags,kernel", [
+    ((1, 3, 64, 224, 224), "relu", "TC"),          # a network's first layer (RGB input), 224 wide
+    ((1, 1, 64, 72, 128), "relu", "TC"),           # one input channel
+    ((2, 5, 130, 20, 24), "skip_pool_relu", "TC_FLAT"),
+    ((1, 7, 200, 14, 14), "relu", "TC_FLAT"),
+])
+@pytest.mark.parametrize("precision", [0, 1])
+def test_tensor_core_few_input_channels(pp, runner, oracle_mod, shape, flags, kernel, precision):
+    """Layers with fewer input channels than one chunk (8, or 16 in fp16): the channels past Ci come
+    from the input box's zero fill and meet zero weights."""
+    N, Ci, Co, H, W = shape
+    rng = np.random.default_rng(Ci * 1000 + Co + precision)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=1.0 if Ci <= 3 else 0.6)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if "skip" in flags else None
+    pool = "pool" in flags
+    g = run_layer(pp, runner, L, x, skip, True, pool, kernel=getattr(pp, "PP_KERNEL_" + kernel),
+                  precision=precision)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, True, pool)
+    check_within(g, y, s, f"{kernel} precision {precision} {shape} {flags}")
 
 
 def test_tensor_core_split_and_tiles(pp, runner, oracle_mod):
@@ -241,6 +263,41 @@ def test_flat_geometry_pin(pp, runner, oracle_mod):
         assert pp.pp_layer_flat_geometry(dl.handle, N, H + 2, W, flags) == (0, 0)
         pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, 0, 0)
         assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, flags) == (0, 0)
+    finally:
+        dl.close()
+
+
+@pytest.mark.parametrize("shape", [(1, 40, 130, 18, 30), (2, 24, 136, 14, 14), (1, 16, 132, 9, 50)])
+@pytest.mark.parametrize("precision", [0, 1])
+def test_flat_geometry_sweep_unaligned_rows(pp, runner, oracle_mod, shape, precision):
+    """Maps whose rows are not 16-byte aligned (W % 4 != 0): the flat kernel stages the tile's rows packed
+    through a tensor map over [N][Ci][H * W] when the planes are aligned and the box fits (at most 256
+    elements), else with per-thread loads; every geometry the planner accepts, both arithmetics."""
+    N, Ci, Co, H, W = shape
+    rng = np.random.default_rng(W * 100 + precision)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.5)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32)
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, True, False)
+    dl = runner.DeviceLayer(L, precision=precision)
+    flags = pp.PP_RELU | pp.PP_ADD_SKIP
+    try:
+        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC_FLAT)
+        accepted = []
+        for R in range(1, 17):
+            for S in (1, 2, 4, 8):
+                try:
+                    pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, R, S)
+                except pp.PPError as e:
+                    assert e.code == pp.PP_ERR_UNSUPPORTED
+                    continue
+                out = torch.full((N, Co, H, W), float("nan"), device="cuda")
+                dl.forward(dev(x), out, dev(skip), N, H, W, flags, torch.cuda.current_stream())
+                torch.cuda.synchronize()
+                assert pp.pp_layer_device_status(dl.handle) == 0
+                check_within(out.cpu().numpy(), y, s, f"{shape} precision {precision} R={R} S={S}")
+                accepted.append((R, S))
+        assert len(accepted) >= 2, accepted
     finally:
         dl.close()
 
@@ -749,12 +806,12 @@ def test_peak_probes(pp):
 F16 = 1  # PP_PRECISION_F16X3
 
 
-@pytest.mark.parametrize("case", [c for c in SMALL if c[1] >= 8])
+@pytest.mark.parametrize("case", SMALL)
 @pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
 @pytest.mark.parametrize("kernel", ["TC", "TC_FLAT"])
 def test_f16_small(pp, runner, oracle_mod, case, flags, kernel):
-    """The fp16-split arithmetic on every small case with at least 8 input channels, both tensor-core
-    kernels (layers with at most 64 filters run the row-tiled kernel for TC_FLAT), every output."""
+    """The fp16-split arithmetic on every small case, both tensor-core kernels (layers with at most 64
+    filters run the row-tiled kernel for TC_FLAT), every output."""
     N, Ci, Co, H, W, P, ring, keep = case
     if flags == "pool_relu" and (H % 2 or W % 2):
         pytest.skip("pool needs even sizes")
