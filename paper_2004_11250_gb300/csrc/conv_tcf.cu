@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   // Offset from the shared array itself (not an integer round trip), so the
   // compiler keeps every access below in the shared state space.
   unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
-  __shared__ __align__(8) uint64_t full[2], wfull[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
+  __shared__ __align__(8) uint64_t full[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
   __shared__ int o_s[FB / 2];    // split phase: original index of each owned filter (-1 beyond Co)
@@ -242,8 +242,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
 
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
-      mbar_init(su32(&full[s]), NLOAD);
-      mbar_init(su32(&wfull[s]), 1);
+      // a stage is full once every loader thread has stored its part of the
+      // input operands and the weight copy (one more arrival, with its bytes)
+      // has landed: the MMA thread waits on one barrier per chunk
+      mbar_init(su32(&full[s]), NLOAD + 1);
       mbar_init(su32(&raw_full[s]), 1);
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
@@ -339,11 +341,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     auto issue_w = [&](int gg, int s) {
       const Tile T = tile_of(p, tile_index(gg / nchm));
       const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c_beg + gg % nchm) * W_BYTES;
-      mbar_arrive_expect_tx(su32(&wfull[s]), W_BYTES);
+      mbar_arrive_expect_tx(su32(&full[s]), W_BYTES);
       asm volatile(
           "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
               su32(smem + (size_t)s * p.stage)),
-          "l"(src), "r"(W_BYTES), "r"(su32(&wfull[s]))
+          "l"(src), "r"(W_BYTES), "r"(su32(&full[s]))
           : "memory");
     };
     int g = 0, w_issued = 0, raw_issued = 0;
@@ -495,12 +497,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     if (F16 && range_bad != 0) atomicOr(p.status, ppc::kStatusF16Range);
     if (tid == 0) {
       // No copy may still be writing shared memory when the CTA exits: wait
-      // (bounded) for the last copies issued into each stage.
+      // (bounded) for the last copies issued into each stage.  (After a timeout
+      // a stage's barrier may lack loader arrivals and never complete; the
+      // bounded wait then outlasts any copy still in flight.)
       for (int gg = raw_issued > 2 ? raw_issued - 2 : 0; gg < raw_issued; ++gg)
         for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&raw_full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
         }
       for (int gg = w_issued > 2 ? w_issued - 2 : 0; gg < w_issued; ++gg)
-        for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&wfull[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+        for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
         }
     }
     __syncwarp();
@@ -516,7 +520,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         bool okc = true;
         for (int c = c_beg; c < c_end; ++c, ++g) {
           const int s = g & 1, use = g >> 1;
-          if (!wait(&full[s], (uint32_t)(use & 1)) || !wait(&wfull[s], (uint32_t)(use & 1))) {
+          if (!wait(&full[s], (uint32_t)(use & 1))) {
             okc = false;
             break;
           }
