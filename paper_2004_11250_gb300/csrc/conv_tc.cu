@@ -189,7 +189,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
   // Offset from the shared array itself (not an integer round trip), so the
   // compiler keeps every access below in the shared state space.
   unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
-  __shared__ __align__(8) uint64_t full[2], wfull[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
+  __shared__ __align__(8) uint64_t full[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
 
@@ -209,12 +209,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
-      mbar_init(su32(&full[s]), NLOAD);
+      // full: every loader thread's operand stores plus the weight copy (one
+      // more arrival, with its bytes), so the MMA thread waits once per chunk
+      mbar_init(su32(&full[s]), NLOAD + 1);
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
       mbar_init(su32(&acc_empty[s]), NEPI);
       mbar_init(su32(&raw_full[s]), 1);
-      mbar_init(su32(&wfull[s]), 1);
     }
     mbar_init(su32(&done_bar), 1);
     abort_s = 0;
@@ -233,7 +234,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 
   if (warp < MMA_WARP) {
     // ------------------------------------------------------------ loaders
-    // Thread 0 issues the copies: weights (bulk, on wfull[s]) and, with a tensor
+    // Thread 0 issues the copies: weights (bulk, on full[s]) and, with a tensor
     // map, the raw input box (on raw_full); all loader threads then transpose the
     // box into the hi / lo operand tiles and arrive on full[s].
     const int nall = nmine * p.nch;  // chunks of this CTA
@@ -255,11 +256,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
     auto issue_w = [&](int gg, int s) {
       const Tile T = tile_of(p, (int)blockIdx.x + (gg / p.nch) * (int)gridDim.x, G::R, TW);
       const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + gg % p.nch) * G::W_BYTES;
-      mbar_arrive_expect_tx(su32(&wfull[s]), G::W_BYTES);
+      mbar_arrive_expect_tx(su32(&full[s]), G::W_BYTES);
       asm volatile(
           "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
               su32(smem + s * G::STAGE)),
-          "l"(src), "r"(G::W_BYTES), "r"(su32(&wfull[s]))
+          "l"(src), "r"(G::W_BYTES), "r"(su32(&full[s]))
           : "memory");
     };
     // The weights do not depend on the previous kernel in the stream: the first
@@ -439,13 +440,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
     if (tid == 0) {
       // No copy may still be writing shared memory when the CTA exits: after an
       // early stop, wait (bounded) for the last copies of each kind to land.
+      // (A stage's barrier may then lack loader arrivals and never complete;
+      // the bounded wait outlasts any copy still in flight.)
       for (int gg = raw_issued - 2; gg < raw_issued; ++gg)
         if (gg >= 0)
           for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&raw_full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
           }
       for (int gg = w_issued - 2; gg < w_issued; ++gg)
         if (gg >= 0)
-          for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&wfull[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+          for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
           }
     }
   } else if (warp == MMA_WARP) {
@@ -460,7 +463,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
         bool okc = true;
         for (int c = 0; c < p.nch; ++c, ++g) {
           const int s = g & 1, use = g >> 1;
-          if (!wait(&full[s], (uint32_t)(use & 1)) || !wait(&wfull[s], (uint32_t)(use & 1))) {
+          if (!wait(&full[s], (uint32_t)(use & 1))) {
             okc = false;
             break;
           }
