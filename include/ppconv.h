@@ -184,7 +184,7 @@ pp_status pp_conv_forward(const pp_layer* layer, const float* x, float* y, const
  *   The first call on a device sets the kernel's launch attributes and should
  *   come before any stream capture.
  * Errors: as pp_conv_forward; PP_ERR_UNSUPPORTED also when the layer cannot
- *   run the flat kernel at this shape (Ci < 8, Co <= 64, W > 128).
+ *   run the flat kernel at this shape (Co <= 64, W > 128).
  */
 pp_status pp_conv_forward_noalloc(const pp_layer* layer, const float* x, float* y, const float* skip, int N, int H,
                                   int W, int flags, void* stream);
@@ -235,7 +235,7 @@ pp_status pp_layer_set_output_order(pp_layer* layer, const int32_t* order, void*
  * bytes of the tf32 one) from a host copy of the packed layer, synchronously
  * on stream; a CUDA graph captured before keeps the old arithmetic.
  * Errors: PP_ERR_INVALID_ARG (unknown precision, NaN bound), PP_ERR_UNSUPPORTED
- * (F16X3 on a layer without a tensor-core layout: Ci < 8), PP_ERR_CUDA,
+ * (F16X3 on a layer without a tensor-core layout), PP_ERR_CUDA,
  * PP_ERR_OOM. */
 #define PP_PRECISION_TF32X3 0
 #define PP_PRECISION_F16X3 1
@@ -247,7 +247,8 @@ pp_status pp_layer_precision(const pp_layer* layer, int* precision, float* input
  * convolution within the documented fp32 bound.
  *   PP_KERNEL_TC        implicit GEMM on the tensor cores over the 9 taps
  *                       (zeros where pruned), 3xTF32 for fp32 accuracy; any
- *                       pattern set; needs Ci >= 8.
+ *                       pattern set; any Ci (channels padded to the
+ *                       chunk of 8, or 16 in fp16, with zeros).
  *   PP_KERNEL_TC_FLAT   the same contraction with whole output rows flattened
  *                       into one MMA and, for layers with few output tiles,
  *                       the input channels split over a thread-block cluster
