@@ -301,9 +301,14 @@ pp_status pp_layer_autotune(pp_layer* layer, int N, int H, int W, int flags, voi
  * for that shape (R rows of round_up(W + 2, 8) pixels must fit one MMA of at
  * most 256 columns, R even when pooling; S a power of 2 up to 16, at most the
  * number of 8-channel chunks, with tiles x S within the SM count and the
- * cluster size launchable on this GPU).  Every geometry stays within the
- * error bound; geometries with different splits group the channel sum
- * differently, so their last bits may differ (each is deterministic). */
+ * cluster size launchable on this GPU).  S | PP_FLAT_PAIRED names the same
+ * split run by CTA pairs: two filter blocks of a tile share each MMA (M = 256
+ * over two SMs, cta_group::2), each SM staging half of the tile's pixels, in
+ * clusters of 2 S CTAs (S up to 8; layers with an even number of 128-filter
+ * blocks).  Every geometry stays within the error bound; geometries with
+ * different splits group the channel sum differently, so their last bits may
+ * differ (each is deterministic). */
+#define PP_FLAT_PAIRED 256
 pp_status pp_layer_flat_geometry(const pp_layer* layer, int N, int H, int W, int flags, int* R, int* S);
 pp_status pp_layer_pin_flat_geometry(pp_layer* layer, int N, int H, int W, int flags, int R, int S);
 

@@ -835,8 +835,8 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
   std::vector<Cand> cand;
   if (L->tc_ok) cand.push_back({PP_KERNEL_TC, 0, 0});
   if (L->tc_ok && L->tc.FB == 128) {
-    int R[4], S[4];
-    const int n = ppc::tcf_plan(L->tc, N, H, W, flags, R, S, 4);
+    int R[6], S[6];
+    const int n = ppc::tcf_plan(L->tc, N, H, W, flags, R, S, 6);
     for (int k = 0; k < n; ++k) cand.push_back({PP_KERNEL_TC_FLAT, R[k], S[k]});
   }
   if (L->tm_ok) cand.push_back({PP_KERNEL_TMEM, 0, 0});

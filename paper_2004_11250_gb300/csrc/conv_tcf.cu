@@ -122,14 +122,16 @@ __device__ __forceinline__ Tile tile_of(const FlatParams& p, int t) {
 // items are 4 adjacent accumulator columns of one filter (pooled: 2 rows x 4
 // columns, i.e. 2 pooled outputs), spread over all threads of the CTA; each
 // item issues its S 16-byte loads before it sums them.
+// The S partials of a tile are in cluster CTAs rofs, rofs + rstride, ... (rstride
+// 2 with CTA pairs: the even and the odd CTAs hold different filter blocks).
 template <int S>
 __device__ __forceinline__ void split_reduce(const FlatParams& p, const Tile& T, int m0, int nm, float* part,
-                                             const int* o_s, const float* b_s, int tid) {
+                                             const int* o_s, const float* b_s, int tid, int rstride, int rofs) {
   namespace cg = cooperative_groups;
   cg::cluster_group cl = cg::this_cluster();
   const float* src[S];
 #pragma unroll
-  for (int s = 0; s < S; ++s) src[s] = cl.map_shared_rank(part, s);
+  for (int s = 0; s < S; ++s) src[s] = cl.map_shared_rank(part, s * rstride + rofs);
   const int pst = p.ncols + 4;
   const bool relu = p.flags & PP_RELU;
   const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
@@ -213,8 +215,16 @@ __device__ __forceinline__ void split_reduce(const FlatParams& p, const Tile& T,
   }
 }
 
-template <bool SPLIT, bool F16>
+// PAIR: the CTAs of a cluster form pairs (cluster ranks 2k, 2k + 1) that run
+// two filter blocks of the same tile and channel range with cta_group::2 MMAs
+// (M = 256): each CTA holds its own block's weights (A) and stages half of
+// the tile's pixels (B columns 0 .. N/2-1 in the even CTA, N/2 .. N-1 in the
+// odd one); the even CTA's MMA thread issues for both, once the odd CTA has
+// reported its stage full, and its commits arrive in both CTAs.  Pairs run in
+// cluster-split mode (one tile per CTA).
+template <bool SPLIT, bool F16, bool PAIR>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
+  static_assert(SPLIT || !PAIR, "CTA pairs run in cluster-split mode");
   constexpr int KCH = F16 ? 16 : KC;  // input channels per chunk
   constexpr int CPH = KCH / 2;         // channels per K half (16 bytes of one pixel row of an operand)
   extern __shared__ unsigned char smem_raw[];
@@ -222,6 +232,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   // compiler keeps every access below in the shared state space.
   unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t full[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
+  __shared__ __align__(8) uint64_t pfull[2];  // PAIR, even CTA: the odd CTA's stage is full
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
   __shared__ int o_s[FB / 2];    // split phase: original index of each owned filter (-1 beyond Co)
@@ -252,33 +263,51 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       mbar_init(su32(&acc_empty[s]), NEPI);
     }
     mbar_init(su32(&done_bar), 1);
+    mbar_init(su32(&pfull[0]), 1);
+    mbar_init(su32(&pfull[1]), 1);
     abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == MMA_WARP) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&tmem_s)),
-                 "n"(2 * NMAX));
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    if (PAIR) {  // both CTAs of the pair allocate together
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&tmem_s)),
+                   "n"(2 * NMAX));
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&tmem_s)),
+                   "n"(2 * NMAX));
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
   }
   tm_fence_before();
   __syncthreads();
   tm_fence_after();
   const uint32_t tmem = tmem_s;
 
-  // This CTA's tiles and channel-chunk range.
+  // This CTA's tiles and channel-chunk range.  Cluster rank crank: split rank
+  // srank, and with pairs the position pp in the pair (0: issues the MMAs).
+  const int csize = PAIR ? 2 * p.split : p.split;
+  const int crank = SPLIT ? (int)blockIdx.x % csize : 0;
+  const int pp = PAIR ? (crank & 1) : 0;
+  const int srank = PAIR ? (crank >> 1) : crank;
   int nmine, c_beg, c_end;
   if (SPLIT) {
-    const int rank = (int)blockIdx.x % p.split;
     nmine = 1;
-    c_beg = rank * p.nch / p.split;
-    c_end = (rank + 1) * p.nch / p.split;
+    c_beg = srank * p.nch / p.split;
+    c_end = (srank + 1) * p.nch / p.split;
   } else {
     nmine = p.ntiles > (int)blockIdx.x ? (p.ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
     c_beg = 0;
     c_end = p.nch;
   }
   auto tile_index = [&](int i) -> int {
-    return SPLIT ? (int)blockIdx.x / p.split : (int)blockIdx.x + i * (int)gridDim.x;
+    return SPLIT ? (int)blockIdx.x / csize : (int)blockIdx.x + i * (int)gridDim.x;
+  };
+  // with pairs a tile index names a pair of filter blocks (p.nfb counts pairs)
+  auto my_tile = [&](int t) -> Tile {
+    Tile T = tile_of(p, t);
+    if (PAIR) T.fb = 2 * T.fb + pp;
+    return T;
   };
   const int brows = p.R + 2;
 
@@ -296,17 +325,20 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       const int it = b * NLOAD + tid;
       const int kh = it >= p.npix ? 1 : 0;
       const int pix = it - kh * p.npix;
-      const int br = pix / p.bcols, bc = pix - br * p.bcols;
-      const bool has = it < 2 * p.npix;
+      // operand row pix holds staged pixel pix (+ N/2 in the odd CTA of a pair);
+      // staged pixels past the box's rows only feed dropped columns: zeros
+      const int sp = PAIR ? pix + pp * (p.ncols >> 1) : pix;
+      const int br = sp / p.bcols, bc = sp - br * p.bcols;
+      const bool has = it < 2 * p.npix, inbox = !PAIR || br < brows;
       // 4-D box: columns from -4, zero filled outside the image.  Packed rows
       // (plane): row br of the tile starts br * W elements into the box (after
       // the tile's alignment shift, added per tile); the halo columns, which
       // the packed rows do not hold, are zeros.
-      roff[b] = !has ? -1
+      roff[b] = !(has && inbox) ? -1
                      : (p.plane ? ((bc >= 1 && bc <= p.W) ? kh * CPH * p.raw_w + br * p.W + bc - 1 : -1)
                                 : (kh * CPH * brows + br) * p.raw_w + bc + 3);
       doff[b] = has ? kh * p.npixa + pix : -1;
-      rowcol[b] = (kh << 30) | (br << 15) | bc;
+      rowcol[b] = (kh << 30) | ((inbox ? br : 0x7FFF) << 15) | bc;  // row 0x7FFF: outside the image
     }
     const int cstride = p.plane ? p.raw_w : brows * p.raw_w;  // between two channels of the box
     // Packed rows: the box starts at element (r0 - 1) W rounded down to a
@@ -317,7 +349,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // zero fill outside the image is the convolution's padding.
     auto issue_raw = [&](int gg, unsigned char* dst) {
       const int i = gg / nchm, c = c_beg + gg % nchm;
-      const Tile T = tile_of(p, tile_index(i));
+      const Tile T = my_tile(tile_index(i));
       mbar_arrive_expect_tx(su32(&raw_full[gg & 1]), (uint32_t)p.raw_bytes);
       if (p.plane) {
         const int x0 = (T.r0 - 1) * p.W - plane_shift(T);
@@ -339,7 +371,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // (as many as the ring has slots), not only once the chunk's stage is free.
     // Weights of chunk gg into stage s (thread 0).
     auto issue_w = [&](int gg, int s) {
-      const Tile T = tile_of(p, tile_index(gg / nchm));
+      const Tile T = my_tile(tile_index(gg / nchm));
       const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c_beg + gg % nchm) * W_BYTES;
       mbar_arrive_expect_tx(su32(&full[s]), W_BYTES);
       asm volatile(
@@ -361,7 +393,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     bool stop = false;  // identical in every loader thread (decided by group_any)
     uint32_t range_bad = 0;  // f16: nonzero once an input is non-finite or overflows fp16 after scaling
     for (int i = 0; i < nmine && !stop; ++i) {
-      const Tile T = tile_of(p, tile_index(i));
+      const Tile T = my_tile(tile_index(i));
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
       const int tsh = plane_shift(T);
       for (int c = c_beg; c < c_end; ++c, ++g) {
@@ -510,7 +542,18 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     __syncwarp();
   } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // (with pairs: in the even CTA; the odd CTA's thread reports its stages full)
+    const uint16_t pmask = (uint16_t)(3u << (crank & ~1));  // PAIR: both CTAs of this pair
+    if (PAIR && lane == 0 && pp == 1) {
+      int g = 0;
+      bool ok = true;
+      for (int c = c_beg; c < c_end && ok; ++c, ++g) {
+        const int s = g & 1, use = g >> 1;
+        ok = wait(&full[s], (uint32_t)(use & 1));
+        if (ok) mbar_arrive_remote(map_rank(su32(&pfull[s]), (uint32_t)(crank ^ 1)));
+      }
+      asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    } else if (lane == 0) {
       int g = 0;
       for (int i = 0; i < nmine && !abort_s; ++i) {
         const int b = i & 1, ub = i >> 1;
@@ -520,7 +563,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         bool okc = true;
         for (int c = c_beg; c < c_end; ++c, ++g) {
           const int s = g & 1, use = g >> 1;
-          if (!wait(&full[s], (uint32_t)(use & 1))) {
+          if (!wait(&full[s], (uint32_t)(use & 1)) || (PAIR && !wait(&pfull[s], (uint32_t)(use & 1)))) {
             okc = false;
             break;
           }
@@ -537,7 +580,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             const uint64_t off = (uint64_t)((t / 3) * p.bcols + t % 3);
             const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * W_TILE / 16);
             const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows
-            if (F16) {
+            if (PAIR) {
+              if (F16) {
+                mma_f16_pair(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+                mma_f16_pair(d + ACC2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+                mma_f16_pair(d + ACC2, whi, xl0 + off, p.idesc, 1u);
+              } else {
+                mma_tf32_pair(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+                mma_tf32_pair(d, wlo, xh0 + off, p.idesc, 1u);
+                mma_tf32_pair(d, whi, xl0 + off, p.idesc, 1u);
+              }
+            } else if (F16) {
               // acc1 += w_hi x_hi; acc2 += w_lo x_hi + w_hi x_lo (both lo parts scaled by 2^11)
               mma_f16(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
               mma_f16(d + ACC2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
@@ -548,16 +601,25 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
               mma_tf32(d, whi, xl0 + off, p.idesc, 1u);
             }
           }
-          mma_commit(su32(&empty[s]));
+          if (PAIR)
+            mma_commit_pair(su32(&empty[s]), pmask);
+          else
+            mma_commit(su32(&empty[s]));
         }
         if (!okc) break;
-        mma_commit(su32(&acc_full[b]));
+        if (PAIR)
+          mma_commit_pair(su32(&acc_full[b]), pmask);
+        else
+          mma_commit(su32(&acc_full[b]));
       }
       // every MMA issued by this thread is complete before TMEM is released
       // the next kernel in the stream may start its prologue (it waits for this
       // grid to complete before it reads anything this grid writes)
       asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-      mma_commit(su32(&done_bar));
+      if (PAIR)
+        mma_commit_pair(su32(&done_bar), pmask);
+      else
+        mma_commit(su32(&done_bar));
       wait(&done_bar, 0u);
     }
     __syncwarp();
@@ -573,7 +635,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       // the whole warp leaves together: its TMEM loads are warp-collective
       if (!__all_sync(0xffffffffu, wait(&acc_full[b], (uint32_t)(ub & 1)))) break;
       tm_fence_after();
-      const Tile T = tile_of(p, tile_index(i));
+      const Tile T = my_tile(tile_index(i));
       const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NMAX);
       const int m = 32 * q + lane;  // filter within the block = TMEM lane
       // f16: the filter's inverse scale (the layout holds nfb x FB entries, padding included)
@@ -709,9 +771,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // This CTA finishes filters [m0, m1) of the tile (at most FB / 2 of them);
     // their original indices and biases are fetched now, so the loads overlap
     // the barrier wait.
-    const int tile = (int)blockIdx.x / p.split, rank = (int)blockIdx.x % p.split;
-    const int m0 = rank * FB / p.split, m1 = (rank + 1) * FB / p.split, nm = m1 - m0;
-    const Tile T = tile_of(p, tile);
+    const int tile = (int)blockIdx.x / csize, rstride = PAIR ? 2 : 1;
+    const int m0 = srank * FB / p.split, m1 = (srank + 1) * FB / p.split, nm = m1 - m0;
+    const Tile T = my_tile(tile);
     if (tid < nm) {
       const int jr = T.fb * FB + m0 + tid;
       o_s[tid] = jr < p.Co ? __ldg(p.perm + jr) : -1;
@@ -722,10 +784,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     if (!abort_s) {
       float* part = reinterpret_cast<float*>(smem);
       switch (p.split) {
-        case 2: split_reduce<2>(p, T, m0, nm, part, o_s, b_s, tid); break;
-        case 4: split_reduce<4>(p, T, m0, nm, part, o_s, b_s, tid); break;
-        case 8: split_reduce<8>(p, T, m0, nm, part, o_s, b_s, tid); break;
-        default: split_reduce<16>(p, T, m0, nm, part, o_s, b_s, tid); break;
+        case 2: split_reduce<2>(p, T, m0, nm, part, o_s, b_s, tid, rstride, pp); break;
+        case 4: split_reduce<4>(p, T, m0, nm, part, o_s, b_s, tid, rstride, pp); break;
+        case 8: split_reduce<8>(p, T, m0, nm, part, o_s, b_s, tid, rstride, pp); break;
+        default: split_reduce<16>(p, T, m0, nm, part, o_s, b_s, tid, rstride, pp); break;
       }
     }
     __syncwarp();
@@ -735,8 +797,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   tm_fence_before();
   __syncthreads();
   tm_fence_after();
-  if (warp == MMA_WARP)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(2 * NMAX));
+  if (warp == MMA_WARP) {
+    if (PAIR)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(2 * NMAX));
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(2 * NMAX));
+  }
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -755,20 +821,30 @@ cudaError_t init_device(int dev) {
   DeviceState& D = g_dev[dev];
   cudaError_t e = cudaDeviceGetAttribute(&D.sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(ppconv_tcf_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(ppconv_tcf_kernel<false, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 SMEM_ALLOC)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 SMEM_ALLOC)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<false, true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 SMEM_ALLOC)) != cudaSuccess ||
-      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SMEM_ALLOC)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                SMEM_ALLOC)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(ppconv_tcf_kernel<true, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 SMEM_ALLOC)) != cudaSuccess)
     return e;
   // then only portable sizes (up to 8) can be used
-  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, false, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
       cudaSuccess)
     cudaGetLastError();
-  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+      cudaSuccess)
+    cudaGetLastError();
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, false, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+      cudaSuccess)
+    cudaGetLastError();
+  if (cudaFuncSetAttribute(ppconv_tcf_kernel<true, true, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
       cudaSuccess)
     cudaGetLastError();
   for (int s = 2; s <= MAX_SPLIT; s *= 2) {
@@ -785,7 +861,7 @@ cudaError_t init_device(int dev) {
     cfg.numAttrs = 1;
     int n = 0;
     // both precisions launch 544 threads, one CTA per SM, with the same shared memory
-    if (cudaOccupancyMaxActiveClusters(&n, ppconv_tcf_kernel<true, false>, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, ppconv_tcf_kernel<true, false, false>, &cfg) != cudaSuccess) {
       cudaGetLastError();
       n = 0;
     }
@@ -812,7 +888,10 @@ DeviceState* prepare() {
 struct FlatGeo {
   int bcols = 0, R = 0, ncols = 0, npix = 0, npixa = 0, raw_w = 0, raw_bytes = 0, tiles_y = 0, ntiles = 0, split = 1;
   int stage = 0, lo_off = 0, sep = 0, raw_off = 0, raw_slot = 0;
+  bool pair = false;  // CTA pairs over two filter blocks (ntiles then counts pairs of blocks)
   double cost = 1e300;
+  // the split as the geometry API reports it (PP_FLAT_PAIRED set for pairs)
+  int code() const { return split | (pair ? PP_FLAT_PAIRED : 0); }
 };
 
 // Geometry of one launch: rows per tile and split, by a model of the time in
@@ -846,52 +925,62 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
       if (R < 2) break;
     }
     ty = (H + R - 1) / R;
-    FlatGeo G;
-    G.bcols = bcols;
-    G.R = R;
-    G.ncols = (R * bcols + 15) / 16 * 16;
-    G.npix = (R + 2) * bcols;
-    G.npixa = G.npix + 16;
-    G.raw_w = bcols + 4;
-    G.raw_bytes = kch * (R + 2) * G.raw_w * 4;
-    G.tiles_y = ty;
-    const int64_t nt = (int64_t)ty * nfb * N;
-    const int in_bytes = (2 * G.npixa * 16 + 127) / 128 * 128;
-    G.raw_slot = (G.raw_bytes + 127) / 128 * 128;
-    G.stage = W_BYTES + 2 * in_bytes;
-    // a ring of two box slots, else one (copied one chunk ahead), else the box lands in the stage
-    G.sep = 2 * G.stage + 2 * G.raw_slot <= SMEM_USE ? 2 : (2 * G.stage + G.raw_slot <= SMEM_USE ? 1 : 0);
-    if (!G.sep) G.stage = W_BYTES + in_bytes + std::max(in_bytes, G.raw_slot);  // the box lands in lo
-    G.lo_off = W_BYTES + in_bytes;
-    G.raw_off = 2 * G.stage;
-    if (G.npixa > PIX_MAX || 2 * G.stage > SMEM_USE || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
-    G.ntiles = (int)nt;
-    const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
-    const double per_chunk = std::max(std::max(mma, W_BYTES / 48.0), 1500.0);
-    for (int s = 1; s <= MAX_SPLIT; s *= 2) {
-      if (s > 1 && (!allow_split || s > nch || D.max_clusters[s] <= 0 || (int64_t)G.ntiles * s > D.sms)) continue;
-      double cost;
-      if (s == 1) {
-        const double waves = std::ceil((double)G.ntiles / D.sms);
-        cost = waves * nch * per_chunk + 5000.0;
-      } else {
-        // clusters beyond those that fit on the GPU at once run in a later wave
-        const double waves = std::ceil((double)G.ntiles / D.max_clusters[s]);
-        cost = waves * (std::ceil((double)nch / s) * per_chunk + 5000.0 + 16.0 * G.ncols);
+    for (int pair = 0; pair < 2; ++pair) {
+      // pairs: two filter blocks per tile, cluster of 2 S, each CTA stages half of the tile's columns
+      if (pair && (!allow_split || (nfb & 1))) continue;
+      FlatGeo G;
+      G.pair = pair != 0;
+      G.bcols = bcols;
+      G.R = R;
+      G.ncols = (R * bcols + 15) / 16 * 16;
+      G.npix = pair ? (G.ncols / 2 + 2 * bcols + 2 + 7) / 8 * 8 : (R + 2) * bcols;
+      G.npixa = G.npix + 16;
+      G.raw_w = bcols + 4;
+      G.raw_bytes = kch * (R + 2) * G.raw_w * 4;
+      G.tiles_y = ty;
+      const int64_t nt = (int64_t)ty * (pair ? nfb / 2 : nfb) * N;
+      const int in_bytes = (2 * G.npixa * 16 + 127) / 128 * 128;
+      G.raw_slot = (G.raw_bytes + 127) / 128 * 128;
+      G.stage = W_BYTES + 2 * in_bytes;
+      // a ring of two box slots, else one (copied one chunk ahead), else the box lands in the stage
+      G.sep = 2 * G.stage + 2 * G.raw_slot <= SMEM_USE ? 2 : (2 * G.stage + G.raw_slot <= SMEM_USE ? 1 : 0);
+      if (!G.sep) G.stage = W_BYTES + in_bytes + std::max(in_bytes, G.raw_slot);  // the box lands in lo
+      G.lo_off = W_BYTES + in_bytes;
+      G.raw_off = 2 * G.stage;
+      if (G.npixa > PIX_MAX || 2 * G.stage > SMEM_USE || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
+      G.ntiles = (int)nt;
+      const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
+      // pairs: each SM reads half the input operand bytes per MMA and issues half the MMAs; modelled as 0.8
+      // of the chunk time (the input operand reads are ~20 % of a chunk's shared-memory traffic)
+      const double per_chunk = std::max(std::max(mma, W_BYTES / 48.0), 1500.0) * (pair ? 0.8 : 1.0);
+      // (split mode owns at most FB / 2 filters per CTA in its second phase: pairs split at least 2 ways)
+      for (int s = pair ? 2 : 1; s <= MAX_SPLIT; s *= 2) {
+        const int cs = pair ? 2 * s : s;  // cluster size
+        if (cs > MAX_SPLIT) break;
+        if (cs > 1 && (!allow_split || s > nch || D.max_clusters[cs] <= 0 || (int64_t)G.ntiles * cs > D.sms)) continue;
+        double cost;
+        if (cs == 1) {
+          const double waves = std::ceil((double)G.ntiles / D.sms);
+          cost = waves * nch * per_chunk + 5000.0;
+        } else {
+          // clusters beyond those that fit on the GPU at once run in a later wave
+          const double waves = std::ceil((double)G.ntiles / D.max_clusters[cs]);
+          cost = waves * (std::ceil((double)nch / s) * per_chunk + 5000.0 + 16.0 * G.ncols);
+        }
+        G.split = s;
+        G.cost = cost;
+        bool dup = false;
+        for (int k = 0; k < n; ++k) dup = dup || (out[k].R == G.R && out[k].code() == G.code());
+        if (dup) continue;
+        // insert in cost order, keeping the best maxn
+        if (n == maxn && out[n - 1].cost <= cost) continue;
+        int k = n < maxn ? n++ : maxn - 1;  // a full list drops its worst entry
+        while (k > 0 && out[k - 1].cost > cost) {
+          out[k] = out[k - 1];
+          --k;
+        }
+        out[k] = G;
       }
-      G.split = s;
-      G.cost = cost;
-      bool dup = false;
-      for (int k = 0; k < n; ++k) dup = dup || (out[k].R == G.R && out[k].split == s);
-      if (dup) continue;
-      // insert in cost order, keeping the best maxn
-      if (n == maxn && out[n - 1].cost <= cost) continue;
-      int k = n < maxn ? n++ : maxn - 1;  // a full list drops its worst entry
-      while (k > 0 && out[k - 1].cost > cost) {
-        out[k] = out[k - 1];
-        --k;
-      }
-      out[k] = G;
     }
   }
   return n;
@@ -908,7 +997,7 @@ bool flat_pick(int N, int H, int W, int nch, int nfb, bool pool, const DeviceSta
   FlatGeo all[160];
   const int n = flat_candidates(N, H, W, nch, nfb, pool, true, D, all, 160, f16);
   for (int k = 0; k < n; ++k)
-    if (all[k].R == R && all[k].split == S) {
+    if (all[k].R == R && all[k].code() == S) {
       *out = all[k];
       return true;
     }
@@ -967,7 +1056,7 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.H = H;
   p.W = W;
   p.nch = f16 ? T.nch16 : T.nch;
-  p.nfb = T.nfb;
+  p.nfb = G.pair ? T.nfb / 2 : T.nfb;  // pairs: the tile index names a pair of filter blocks
   p.flags = flags;
   p.bcols = G.bcols;
   p.R = G.R;
@@ -984,7 +1073,8 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.tiles_y = G.tiles_y;
   p.ntiles = G.ntiles;
   p.split = G.split;
-  p.idesc = f16 ? idesc_f16(FB, G.ncols) : idesc_tf32(FB, G.ncols);
+  const int mrows = G.pair ? 2 * FB : FB;  // pairs: one M = 256 MMA over both CTAs' filter blocks
+  p.idesc = f16 ? idesc_f16(mrows, G.ncols) : idesc_tf32(mrows, G.ncols);
   CUtensorMap xmap;
   std::memset(&xmap, 0, sizeof(xmap));
   p.use_tma = 0;
@@ -1033,19 +1123,28 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   cfg.dynamicSmemBytes = SMEM_ALLOC;
   cfg.stream = stream;
   cudaError_t e;
-  if (G.split > 1) {
+  if (G.pair) {
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = (unsigned)(2 * G.split);
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
+    cfg.gridDim = dim3((unsigned)(G.ntiles * 2 * G.split));
+    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, true, true>, p, xmap)
+            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, false, true>, p, xmap);
+  } else if (G.split > 1) {
     at[1].id = cudaLaunchAttributeClusterDimension;
     at[1].val.clusterDim.x = (unsigned)G.split;
     at[1].val.clusterDim.y = 1;
     at[1].val.clusterDim.z = 1;
     cfg.numAttrs = 2;
     cfg.gridDim = dim3((unsigned)(G.ntiles * G.split));
-    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, true>, p, xmap)
-            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, false>, p, xmap);
+    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, true, false>, p, xmap)
+            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<true, false, false>, p, xmap);
   } else {
     cfg.gridDim = dim3((unsigned)std::min(G.ntiles, D->sms));
-    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false, true>, p, xmap)
-            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false, false>, p, xmap);
+    e = f16 ? cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false, true, false>, p, xmap)
+            : cudaLaunchKernelEx(&cfg, ppconv_tcf_kernel<false, false, false>, p, xmap);
   }
   if (e != cudaSuccess) {
     cudaGetLastError();
@@ -1067,7 +1166,7 @@ int tcf_plan(const TcLayout& T, int N, int H, int W, int flags, int* R, int* S, 
                                 std::min(maxn, 16), T.f16);
   for (int k = 0; k < n; ++k) {
     R[k] = G[k].R;
-    S[k] = G[k].split;
+    S[k] = G[k].code();
   }
   return n;
 }

@@ -48,6 +48,7 @@ PP_PROBE_MMA_F16 = 2
 
 PP_PRECISION_TF32X3 = 0
 PP_PRECISION_F16X3 = 1
+PP_FLAT_PAIRED = 256  # or-ed into a flat-kernel split: CTA pairs over two filter blocks
 
 PP_STATUS_TIMEOUT = 1
 PP_STATUS_F16_RANGE = 2

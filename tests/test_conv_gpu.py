@@ -245,7 +245,7 @@ def test_flat_geometry_pin(pp, runner, oracle_mod):
         assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, flags) == (0, 0)
         accepted = []
         for R in range(1, 17):
-            for S in (1, 2, 4, 8, 16):
+            for S in (1, 2, 4, 8, 16) + tuple(pp.PP_FLAT_PAIRED | s for s in (1, 2, 4, 8)):
                 try:
                     pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, R, S)
                 except pp.PPError as e:
@@ -258,11 +258,63 @@ def test_flat_geometry_pin(pp, runner, oracle_mod):
                 check_within(out.cpu().numpy(), y, s, f"flat geometry R={R} S={S}")
                 accepted.append((R, S))
         assert len(accepted) >= 3 and any(S > 1 for _, S in accepted), accepted
+        assert any(S & pp.PP_FLAT_PAIRED for _, S in accepted), accepted  # 130 filters: two blocks, a pair
         assert all(R % 2 == 0 for R, _ in accepted)  # pooling needs row pairs
         # another shape's pin is not reported for this one; R = 0 unpins
         assert pp.pp_layer_flat_geometry(dl.handle, N, H + 2, W, flags) == (0, 0)
         pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, 0, 0)
         assert pp.pp_layer_flat_geometry(dl.handle, N, H, W, flags) == (0, 0)
+    finally:
+        dl.close()
+
+
+PAIR_CASES = [
+    # N, Ci, Co, H, W, flags: filter blocks in pairs (cta_group::2), every accepted paired geometry
+    (1, 136, 256, 28, 28, "relu"),
+    (1, 72, 512, 14, 14, "pool_relu"),
+    (2, 40, 250, 20, 30, "skip_relu"),   # the second block ragged (122 filters)
+    (1, 24, 384, 8, 126, "none"),        # three filter blocks: no pairs
+    (1, 64, 256, 56, 56, "skip_pool_relu"),
+]
+
+
+@pytest.mark.parametrize("case", PAIR_CASES)
+@pytest.mark.parametrize("precision", [0, 1])
+def test_flat_kernel_cta_pairs(pp, runner, oracle_mod, case, precision):
+    """The flat kernel with two filter blocks per MMA over a CTA pair (M = 256, each SM staging half of the
+    tile's columns), at every paired geometry the planner accepts, against the oracle (every output)."""
+    N, Ci, Co, H, W, flags = case
+    rng = np.random.default_rng(Co + W + precision)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.35)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if "skip" in flags else None
+    relu, pool = "relu" in flags, "pool" in flags
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, relu, pool)
+    f = (pp.PP_RELU if relu else 0) | (pp.PP_POOL2 if pool else 0) | (pp.PP_ADD_SKIP if skip is not None else 0)
+    Ho, Wo = (H // 2, W // 2) if pool else (H, W)
+    dl = runner.DeviceLayer(L, precision=precision)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC_FLAT)
+        accepted = []
+        for R in range(1, 17):
+            for S in (1, 2, 4, 8):
+                try:
+                    pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, f, R, pp.PP_FLAT_PAIRED | S)
+                except pp.PPError as e:
+                    assert e.code == pp.PP_ERR_UNSUPPORTED
+                    continue
+                for rep in range(2):  # twice: the pair's barriers and TMEM are set up afresh each launch
+                    out = torch.full((N, Co, Ho, Wo), float("nan"), device="cuda")
+                    dl.forward(dev(x), out, None if skip is None else dev(skip), N, H, W, f,
+                               torch.cuda.current_stream())
+                    torch.cuda.synchronize()
+                    assert pp.pp_layer_device_status(dl.handle) == 0
+                    check_within(out.cpu().numpy(), y, s, f"{case} precision {precision} pair R={R} S={S} #{rep}")
+                accepted.append((R, S))
+        if Co == 384:
+            assert accepted == []
+        else:
+            assert accepted, "no paired geometry accepted"
     finally:
         dl.close()
 
@@ -285,7 +337,7 @@ def test_flat_geometry_sweep_unaligned_rows(pp, runner, oracle_mod, shape, preci
         pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC_FLAT)
         accepted = []
         for R in range(1, 17):
-            for S in (1, 2, 4, 8):
+            for S in (1, 2, 4, 8) + tuple(pp.PP_FLAT_PAIRED | s for s in (1, 2, 4, 8)):
                 try:
                     pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, flags, R, S)
                 except pp.PPError as e:
