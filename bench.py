@@ -355,11 +355,12 @@ def time_graph_of_launches(dn, acts, reps, steps, stream):
     return e0.elapsed_time(e1) / (steps * reps)
 
 
-def traffic_from_profile(kernel_hash: str, kernel: str = None):
-    """Per-launch DRAM bytes (read + write) from the committed ncu summary of the VGG-16 frame, of one
-    kernel (average over its launches in the frame) or of all the frame's convs, if that summary was
-    taken on the current kernel source."""
-    path = os.path.join(ROOT, "profiles", "ppconv_vgg16_dram_traffic.txt")
+def traffic_from_profile(kernel_hash: str, kernel: str = None, precision: str = "tf32x3"):
+    """Per-launch DRAM bytes (read + write) from the committed ncu summary of the VGG-16 frame in this
+    tensor-core arithmetic, of one kernel (average over its launches in the frame) or of all the frame's
+    convs, if that summary was taken on the current kernel source."""
+    name = "ppconv_vgg16_dram_traffic.txt" if precision == "tf32x3" else f"ppconv_vgg16_dram_traffic_{precision}.txt"
+    path = os.path.join(ROOT, "profiles", name)
     try:
         kv = {}
         for line in open(path):
@@ -691,7 +692,9 @@ def main():
     dom_ops = [k for k in pruned if kern[k] == dom]
     achieved = by_kern[dom][0] / by_kern[dom][1] / 1e12
     achieved_alone = sum(shapes[k]["flops"] for k in dom_ops) / (sum(op_ms_alone[k] for k in dom_ops) * 1e-3) / 1e12
-    traffic = traffic_from_profile(kernel_source_hash(), dom)
+    traffic = traffic_from_profile(kernel_source_hash(), dom, args.precision)
+    # the dominant kernel's compulsory bytes per launch (its ops' inputs, outputs and compact weights)
+    algo_bytes = sum(shapes[k]["bytes"] for k in dom_ops) / len(dom_ops)
     # the same op times scaled so that they add up to the graph frame (the events above break the overlap
     # of consecutive ops that programmatic dependent launch gives inside the graph): an apportioned view
     scale = ms_per_step / sum(op_ms)
@@ -757,6 +760,7 @@ def main():
             "gpu_launches": len(spec.ops) * args.steps,
             "roofline": {"bound": "alu", "achieved": round(achieved, 3), "peak": round(FP32_PEAK_TFLOPS, 2),
                          "unit": "TFLOP/s", "frac": round(achieved / FP32_PEAK_TFLOPS, 4), "traffic": traffic,
+                         "algorithmic_bytes": int(algo_bytes),
                          "frac_of_derived_peak": round(achieved / peaks["derived_fp32_tflops"], 4),
                          "kernel": f"{dom} ({len(dom_ops)} of the {len(pruned)} pruned convs, "
                                    f"{100 * by_kern[dom][1] / kt:.0f}% of their in-frame device time)",
@@ -777,7 +781,7 @@ def main():
                                    "timing": "each op launched alone, L2 flushed before every launch"},
                          "all_pruned_ops": {"achieved": round(achieved_all, 3),
                                             "frac": round(achieved_all / FP32_PEAK_TFLOPS, 4),
-                                            "traffic": traffic_from_profile(kernel_source_hash()),
+                                            "traffic": traffic_from_profile(kernel_source_hash(), None, args.precision),
                                             "kernels": sorted(by_kern)},
                          "tensor": tensor,
                          "peak_source": (f"measured: pp_peak_probe FFMA, {peaks['fp32_ffma']['tflops']} TFLOP/s at "
