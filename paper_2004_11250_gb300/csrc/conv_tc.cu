@@ -23,7 +23,9 @@
 // issues the MMAs, warps 9-16 are the epilogue.  The K loop runs over
 // 8-channel chunks, double buffered:
 //   * weights for the chunk, 9 taps x {hi, lo} x (FB x 8) in the canonical
-//     K-major layout, arrive by one bulk async copy (mbarrier transaction count);
+//     K-major layout, arrive by one bulk async copy whose transaction count
+//     completes on the stage's full barrier with the loaders' arrivals, so the
+//     MMA thread waits once per chunk;
 //   * the input box for the chunk (tile rows + 2, columns + halo, 8 channels;
 //     zero fill outside the image is the padding) arrives by a tensor-map copy
 //     (per-thread loads when x is not 16-byte aligned or W % 4 != 0), and the

@@ -26,6 +26,11 @@
 // distributed shared memory, adds them in rank order (deterministic), then
 // bias, skip, ReLU, pool, and stores y.  No global workspace is used.
 //
+// CTA pairs (geometries S | PP_FLAT_PAIRED): the two filter blocks of a tile
+// run on two CTAs of a cluster as one M = 256 MMA (cta_group::2), each CTA
+// holding its own block's weights and staging half of the tile's columns; the
+// even CTA issues every MMA (see the kernel's PAIR parameter).
+//
 // Precision: 3xTF32 (as conv_tc.cu), or, for layers set to PP_PRECISION_F16X3,
 // an fp16 split (F16 instantiations): each operand v is held as hi = f16(v) and
 // lo = f16((v - hi) * 2^11), the weights scaled per filter and the input per
@@ -38,8 +43,10 @@
 // scaling (|x s| >= 65520) or are not finite are flagged by the loaders in the
 // device status word.
 //
-// Roles (17 warps, one CTA per SM): warps 0-7 stage the operands, warp 8
-// allocates TMEM and one of its threads issues the MMAs, warps 9-16 are the
+// Roles (17 warps, one CTA per SM): warps 0-7 stage the operands (thread 0
+// also issues the weight and input-box copies), warp 8 allocates TMEM and one
+// of its threads issues the MMAs, waiting once per chunk (the stage's full
+// barrier counts the loaders and the weight copy), warps 9-16 are the
 // epilogue (two per TMEM lane quadrant).  Without a split the CTA is persistent
 // over tiles with two TMEM accumulator buffers, so a tile's epilogue overlaps
 // the next tile's MMAs.  Every mbarrier wait is bounded; a timeout sets the
