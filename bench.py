@@ -375,13 +375,25 @@ def traffic_from_profile(kernel_hash: str, kernel: str = None, precision: str = 
         return None
 
 
+def code_lines(text: str) -> str:
+    """The source without its // comments and blank lines (the sources use no // inside strings)."""
+    out = []
+    for line in text.splitlines():
+        k = line.find("//")
+        line = (line if k < 0 else line[:k]).rstrip()
+        if line:
+            out.append(line)
+    return "\n".join(out)
+
+
 def kernel_source_hash():
-    """sha256 over the conv kernel sources (a profile taken on other sources is stale)."""
+    """sha256 over the conv kernel sources' code, comments left out (a profile taken on other code is
+    stale; an edit of a comment does not change the kernels)."""
     import hashlib
     h = hashlib.sha256()
     for name in ("conv.cu", "conv_tm.cu", "conv_tc.cu", "conv_tcf.cu", "conv_direct.cu", "tc_ptx.cuh", "internal.h"):
-        with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2004_11250_gb300", "csrc", name), encoding="utf-8") as f:
+            h.update(code_lines(f.read()).encode())
     return h.hexdigest()
 
 
