@@ -828,7 +828,7 @@ extern "C" pp_status pp_layer_autotune(pp_layer* L, int N, int H, int W, int fla
   if ((flags & PP_POOL2) && ((H & 1) || (W & 1))) return PP_ERR_UNSUPPORTED;
   cudaStream_t stream = (cudaStream_t)stream_;
   // Candidates: (kernel, flat-kernel rows per tile, split); the flat kernel is
-  // tried at the few best geometries of its cost model.
+  // tried at the six best geometries of its cost model (CTA pairs included).
   struct Cand {
     int kernel, R, S;
   };
