@@ -187,6 +187,8 @@ __device__ __forceinline__ Tile tile_of(const TcParams& p, int t, int R, int TW)
 template <int ORI, int TW, int FB, bool F16>
 __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p, const __grid_constant__ CUtensorMap xmap) {
   using G = Geo<ORI, TW, FB, F16>;
+  // slots of the box ring (its uses sit behind G::SEP; 1 keeps the modulo defined where the ring is absent)
+  constexpr int RING = G::NRAW > 0 ? G::NRAW : 1;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // Offset from the shared array itself (not an integer round trip), so the
   // compiler keeps every access below in the shared state space.
@@ -293,7 +295,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             stop = true;
             break;
           }
-          const float* raw = reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % G::NRAW) * G::RAW);
+          const float* raw = reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % RING) * G::RAW);
 #pragma unroll
           for (int b = 0; b < EI; ++b) {
             const int it = b * NLOAD + tid;
@@ -311,7 +313,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           group_sync<NLOAD>();
           if (tid == 0 && raw_issued < nall && raw_issued == g + G::NRAW) {
-            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % G::NRAW) * G::RAW);
+            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % RING) * G::RAW);
             ++raw_issued;
           }
         }
@@ -348,7 +350,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             stop = true;
             break;
           }
-          const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % G::NRAW) * G::RAW)
+          const float* raw = G::SEP ? reinterpret_cast<const float*>(smem + G::RAW_OFF + (g % RING) * G::RAW)
                                     : reinterpret_cast<const float*>(lo);
           float v[G::ITEMS][G::CPH];
 #pragma unroll
@@ -367,7 +369,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           if (G::SEP) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           group_sync<NLOAD>();  // every raw value is in registers before its slot is reused
           if (G::SEP && tid == 0 && raw_issued < nall && raw_issued == g + G::NRAW) {
-            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % G::NRAW) * G::RAW);
+            issue_raw(raw_issued, smem + G::RAW_OFF + (raw_issued % RING) * G::RAW);
             ++raw_issued;
           }
 #pragma unroll
