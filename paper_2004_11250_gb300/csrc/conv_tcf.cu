@@ -76,10 +76,15 @@ constexpr int NLOAD = 256;            // loader threads (warps 0-7)
 constexpr int MMA_WARP = 8;
 constexpr int EPI_WARP0 = 9;          // warps 9-16
 constexpr int NEPI = 256;
-constexpr int NTHREADS = 544;
+constexpr int WPROD_WARP = 17;        // the weight producer
+constexpr int NTHREADS = 576;
 constexpr int WMAX = 128;             // widest map handled
 constexpr int W_TILE = FB * KC * 4;   // one tap, hi or lo: 128 x 8 fp32 (or 128 x 16 f16)
-constexpr int W_BYTES = NTAP * 2 * W_TILE;
+constexpr int TAP_BYTES = 2 * W_TILE;          // one tap's hi and lo rows
+constexpr int W_BYTES = NTAP * TAP_BYTES;        // the weights of one chunk
+constexpr int NGRP = 3;                          // weight groups per chunk (3 taps each)
+constexpr int GRP_BYTES = W_BYTES / NGRP;        // a slot of the weight ring
+constexpr int WSL_MAX = 7;                       // slots of the weight ring (7, else 6 when short of space)
 constexpr int PIX_MAX = 544;          // staged pixels per K half, padding included
 constexpr int IN_MAX = 2 * PIX_MAX * 16;  // largest hi (or lo) operand of one chunk
 constexpr int SMEM_ALLOC = 231424;    // dynamic shared memory (static use stays below 1 KB)
@@ -88,6 +93,7 @@ constexpr int ITEMS_MAX = (2 * PIX_MAX + NLOAD - 1) / NLOAD;  // (K half, pixel)
 constexpr long WAIT_LIMIT = PP_WAIT_POLLS;  // mbarrier polls before a wait gives up
 constexpr int MAX_SPLIT = 16;
 static_assert(2 * (W_BYTES + 2 * IN_MAX) <= SMEM_USE, "shared memory plan");
+static_assert(GRP_BYTES % 1024 == 0, "weight-ring slots keep 1024-byte alignment");
 static_assert(FB * NMAX * 4 <= SMEM_USE, "split reduction buffer");
 
 struct FlatParams {
@@ -103,7 +109,8 @@ struct FlatParams {
   int N, Ci, Co, H, W;
   int nch, nfb, flags, use_tma;
   int bcols, R, ncols, npix, npixa, raw_w, raw_bytes;
-  int stage, lo_off;        // bytes per stage; offset of the lo operand in a stage (hi is at W_BYTES)
+  int wsl;                  // slots of the weight ring (6 or 7 groups of 3 taps) at the start of shared memory
+  int xoff, xstage, lo_off; // input operand stage s at xoff + s * xstage: hi, then lo at lo_off
   int sep, raw_off, raw_slot;  // input boxes in a ring of their own: sep (2 or 1) slots at raw_off; 0 = none
                                // (slot of chunk g: g & (sep - 1))
   int plane;                // box over x viewed as [N][Ci][H * W]: the staged rows packed, raw_w = box width
@@ -239,6 +246,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   // compiler keeps every access below in the shared state space.
   unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t full[2], raw_full[2], empty[2], acc_full[2], acc_empty[2], done_bar;
+  __shared__ __align__(8) uint64_t wempty[WSL_MAX];  // a weight-ring slot has been read by its MMAs
   __shared__ __align__(8) uint64_t pfull[2];  // PAIR, even CTA: the odd CTA's stage is full
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
@@ -261,15 +269,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
       // a stage is full once every loader thread has stored its part of the
-      // input operands and the weight copy (one more arrival, with its bytes)
-      // has landed: the MMA thread waits on one barrier per chunk
-      mbar_init(su32(&full[s]), NLOAD + 1);
+      // input operands and the chunk's three weight-group copies (three more
+      // arrivals, with their bytes) have landed: the MMA thread waits on one
+      // barrier per chunk
+      mbar_init(su32(&full[s]), NLOAD + NGRP);
       mbar_init(su32(&raw_full[s]), 1);
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
       mbar_init(su32(&acc_empty[s]), NEPI);
     }
     mbar_init(su32(&done_bar), 1);
+    for (int k = 0; k < WSL_MAX; ++k) mbar_init(su32(&wempty[k]), 1);
     mbar_init(su32(&pfull[0]), 1);
     mbar_init(su32(&pfull[1]), 1);
     abort_s = 0;
@@ -376,23 +386,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     };
     // With a ring of their own the boxes are copied one or two chunks ahead of use
     // (as many as the ring has slots), not only once the chunk's stage is free.
-    // Weights of chunk gg into stage s (thread 0).
-    auto issue_w = [&](int gg, int s) {
-      const Tile T = my_tile(tile_index(gg / nchm));
-      const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c_beg + gg % nchm) * W_BYTES;
-      mbar_arrive_expect_tx(su32(&full[s]), W_BYTES);
-      asm volatile(
-          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-              su32(smem + (size_t)s * p.stage)),
-          "l"(src), "r"(W_BYTES), "r"(su32(&full[s]))
-          : "memory");
-    };
-    int g = 0, w_issued = 0, raw_issued = 0;
-    // The weights do not depend on the previous kernel in the stream: the first
-    // two chunks' copies start before waiting for it (programmatic dependent
-    // launch), everything that reads x comes after the wait.
-    if (tid == 0)
-      for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
+    int g = 0, raw_issued = 0;
+    // Everything that reads x comes after the wait for the previous kernel in
+    // the stream (programmatic dependent launch).
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && p.sep)
       for (; raw_issued < p.sep && raw_issued < nall; ++raw_issued)
@@ -414,7 +410,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         // chunk's weight copy, issued once the stage is free).
         // v holds an item's input values, or (f16, split early) its packed hi words then lo words
         float v[ITEMS_MAX][CPH];
-        const bool early = F16 && p.use_tma && p.sep;
+        const bool early = p.use_tma && p.sep;
         if (early) {
           if (group_any<NLOAD>(!wait(&raw_full[s], (uint32_t)(use & 1)))) {
             stop = true;
@@ -469,14 +465,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
           stop = true;
           break;
         }
-        unsigned char* st = smem + (size_t)s * p.stage;
-        float4* hi = reinterpret_cast<float4*>(st + W_BYTES);
+        unsigned char* st = smem + p.xoff + (size_t)s * p.xstage;
+        float4* hi = reinterpret_cast<float4*>(st);
         float4* lo = reinterpret_cast<float4*>(st + p.lo_off);
         if (tid == 0) {
-          if (g >= 2) {
-            issue_w(g, s);
-            ++w_issued;
-          }
           if (p.use_tma && !p.sep) {
             issue_raw(g, reinterpret_cast<unsigned char*>(lo));  // lands in the lo operand, split in place below
             ++raw_issued;
@@ -542,9 +534,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       for (int gg = raw_issued > 2 ? raw_issued - 2 : 0; gg < raw_issued; ++gg)
         for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&raw_full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
         }
-      for (int gg = w_issued > 2 ? w_issued - 2 : 0; gg < w_issued; ++gg)
-        for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
-        }
     }
     __syncwarp();
   } else if (warp == MMA_WARP) {
@@ -561,7 +550,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       }
       asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     } else if (lane == 0) {
-      int g = 0;
+      int g = 0, wslot = 0;  // chunk count and the weight-ring slot of the next group
       for (int i = 0; i < nmine && !abort_s; ++i) {
         const int b = i & 1, ub = i >> 1;
         if (ub > 0 && !wait(&acc_empty[b], (uint32_t)((ub - 1) & 1))) break;
@@ -575,18 +564,25 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
             break;
           }
           tm_fence_after();
-          const unsigned char* st = smem + (size_t)s * p.stage;
+          const unsigned char* st = smem + p.xoff + (size_t)s * p.xstage;
           // descriptors hold address / 16 in their low 14 bits (operands lie below
           // 256 KB), so moving an operand by k pixels of 16 bytes adds k
-          const uint64_t w0 = smem_desc(su32(st), 2 * FB * 16);  // hi and lo rows of a tap in each K half
-          const uint64_t xh0 = smem_desc(su32(st + W_BYTES), (uint32_t)p.npixa * 16);
+          const uint64_t xh0 = smem_desc(su32(st), (uint32_t)p.npixa * 16);
           const uint64_t xl0 = smem_desc(su32(st + p.lo_off), (uint32_t)p.npixa * 16);
+          // the chunk's three weight groups: consecutive slots of the ring
+          int gs[NGRP];
+#pragma unroll
+          for (int k = 0; k < NGRP; ++k) {
+            gs[k] = wslot;
+            wslot = wslot + 1 == p.wsl ? 0 : wslot + 1;
+          }
           const uint32_t acc0 = c == c_beg ? 0u : 1u;  // the range's first chunk overwrites the accumulators
 #pragma unroll
           for (int t = 0; t < NTAP; ++t) {
             const uint64_t off = (uint64_t)((t / 3) * p.bcols + t % 3);
-            const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * W_TILE / 16);
-            const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows
+            // hi and lo rows of a tap in each K half; lo rows follow the hi rows
+            const uint64_t whi = smem_desc(su32(smem + (size_t)gs[t / 3] * GRP_BYTES + (t % 3) * TAP_BYTES), 2 * FB * 16);
+            const uint64_t wlo = whi + (uint64_t)FB;
             if (PAIR) {
               if (F16) {
                 mma_f16_pair(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
@@ -606,6 +602,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
               mma_tf32(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
               mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
               mma_tf32(d, whi, xl0 + off, p.idesc, 1u);
+            }
+            if (t % 3 == 2) {  // the group's slot is free for the producer once these MMAs complete
+              if (PAIR)
+                mma_commit_pair(su32(&wempty[gs[t / 3]]), pmask);
+              else
+                mma_commit(su32(&wempty[gs[t / 3]]));
             }
           }
           if (PAIR)
@@ -628,6 +630,51 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       else
         mma_commit(su32(&done_bar));
       wait(&done_bar, 0u);
+    }
+    __syncwarp();
+  } else if (warp == WPROD_WARP) {
+    // ------------------------------------------------------------ weight producer
+    // A chunk's weights are three groups of 3 tap tiles (24 KB each), copied
+    // into a ring of p.wsl slots.  Group k of a chunk is copied as soon as the
+    // MMAs of the group that held its slot before have completed; with 7 slots
+    // (2 1/3 chunks) the last group of chunk g is copied while the MMAs of
+    // chunk g - 2 still run, not only once they all have.  The three copies
+    // arrive (with their bytes) on the stage's full barrier, so the MMA thread
+    // still waits once per chunk; the copies of chunk g go out only after the
+    // barrier's previous phase (chunk g - 2) has completed.
+    if (lane == 0) {
+      const int nchm = c_end - c_beg;
+      const int nall = nmine * nchm;
+      int slot = 0, use = 0, issued = 0;  // ring position, its round, groups issued
+      bool ok = true;
+      for (int gg = 0; gg < nall && ok; ++gg) {
+        const int s = gg & 1;
+        if (gg >= 2) ok = wait(&full[s], (uint32_t)(((gg - 2) >> 1) & 1));
+        const Tile T = my_tile(tile_index(gg / nchm));
+        const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c_beg + gg % nchm) * W_BYTES;
+        for (int k = 0; k < NGRP && ok; ++k) {
+          if (use > 0) ok = wait(&wempty[slot], (uint32_t)((use - 1) & 1));
+          if (!ok) break;
+          mbar_arrive_expect_tx(su32(&full[s]), GRP_BYTES);
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                  su32(smem + (size_t)slot * GRP_BYTES)),
+              "l"(src + (size_t)k * GRP_BYTES), "r"(GRP_BYTES), "r"(su32(&full[s]))
+              : "memory");
+          ++issued;
+          if (++slot == p.wsl) {
+            slot = 0;
+            ++use;
+          }
+        }
+      }
+      // No copy may still be writing shared memory when the CTA exits: wait
+      // (bounded) for the last two chunks' barriers (after a timeout a
+      // barrier may lack loader arrivals; the bounded wait outlasts any copy).
+      const int last = (issued + NGRP - 1) / NGRP;  // chunks with at least one group issued
+      for (int gg = last > 2 ? last - 2 : 0; gg < last; ++gg)
+        for (long w = 0; w < WAIT_LIMIT && !mbar_try(su32(&full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++w) {
+        }
     }
     __syncwarp();
   } else {
@@ -894,7 +941,7 @@ DeviceState* prepare() {
 
 struct FlatGeo {
   int bcols = 0, R = 0, ncols = 0, npix = 0, npixa = 0, raw_w = 0, raw_bytes = 0, tiles_y = 0, ntiles = 0, split = 1;
-  int stage = 0, lo_off = 0, sep = 0, raw_off = 0, raw_slot = 0;
+  int wsl = 0, xoff = 0, xstage = 0, lo_off = 0, sep = 0, raw_off = 0, raw_slot = 0;
   bool pair = false;  // CTA pairs over two filter blocks (ntiles then counts pairs of blocks)
   double cost = 1e300;
   // the split as the geometry API reports it (PP_FLAT_PAIRED set for pairs)
@@ -948,13 +995,19 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
       const int64_t nt = (int64_t)ty * (pair ? nfb / 2 : nfb) * N;
       const int in_bytes = (2 * G.npixa * 16 + 127) / 128 * 128;
       G.raw_slot = (G.raw_bytes + 127) / 128 * 128;
-      G.stage = W_BYTES + 2 * in_bytes;
-      // a ring of two box slots, else one (copied one chunk ahead), else the box lands in the stage
-      G.sep = 2 * G.stage + 2 * G.raw_slot <= SMEM_USE ? 2 : (2 * G.stage + G.raw_slot <= SMEM_USE ? 1 : 0);
-      if (!G.sep) G.stage = W_BYTES + in_bytes + std::max(in_bytes, G.raw_slot);  // the box lands in lo
-      G.lo_off = W_BYTES + in_bytes;
-      G.raw_off = 2 * G.stage;
-      if (G.npixa > PIX_MAX || 2 * G.stage > SMEM_USE || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
+      // shared memory: the weight ring (7 groups of 3 taps, else 6), two input operand stages (hi, lo),
+      // and a ring of two input-box slots, else one (copied one chunk ahead), else the box lands in lo
+      G.xstage = 2 * in_bytes;
+      G.lo_off = in_bytes;
+      const auto fits = [&](int wsl, int sep) {
+        return wsl * GRP_BYTES + 2 * G.xstage + sep * G.raw_slot <= SMEM_USE;
+      };
+      G.sep = fits(6, 2) ? 2 : (fits(6, 1) ? 1 : 0);
+      if (!G.sep) G.xstage = in_bytes + std::max(in_bytes, G.raw_slot);
+      G.wsl = fits(WSL_MAX, G.sep) ? WSL_MAX : 6;
+      G.xoff = G.wsl * GRP_BYTES;
+      G.raw_off = G.xoff + 2 * G.xstage;
+      if (G.npixa > PIX_MAX || !fits(G.wsl, G.sep) || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
       G.ntiles = (int)nt;
       const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
       // pairs: each SM reads half the input operand bytes per MMA and issues half the MMAs; modelled as 0.8
@@ -1072,7 +1125,9 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.npixa = G.npixa;
   p.raw_w = G.raw_w;
   p.raw_bytes = G.raw_bytes;
-  p.stage = G.stage;
+  p.wsl = G.wsl;
+  p.xoff = G.xoff;
+  p.xstage = G.xstage;
   p.lo_off = G.lo_off;
   p.sep = G.sep;
   p.raw_off = G.raw_off;
