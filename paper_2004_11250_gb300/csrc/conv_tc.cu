@@ -20,12 +20,15 @@
 // Per CTA (17 warps, one CTA per SM, persistent over tiles): warps 0-7 stage
 // the operands, warp 8 owns the TMEM (two accumulator buffers of 256 columns,
 // so one tile's epilogue overlaps the next tile's MMAs) and one of its threads
-// issues the MMAs, warps 9-16 are the epilogue.  The K loop runs over
-// 8-channel chunks, double buffered:
+// issues the MMAs, warps 9-16 are the epilogue; tf32 128-filter tiles add warp
+// 17, which produces the weights.  The K loop runs over 8-channel chunks,
+// double buffered:
 //   * weights for the chunk, 9 taps x {hi, lo} x (FB x 8) in the canonical
-//     K-major layout, arrive by one bulk async copy whose transaction count
-//     completes on the stage's full barrier with the loaders' arrivals, so the
-//     MMA thread waits once per chunk;
+//     K-major layout, arrive by bulk async copies whose transaction counts
+//     complete on the stage's full barrier with the loaders' arrivals, so the
+//     MMA thread waits once per chunk: most tiles copy them whole into the
+//     stage; tf32 128-filter tiles copy them in three groups of 3 taps into a
+//     ring of group slots, each slot refilled as soon as its MMAs complete;
 //   * the input box for the chunk (tile rows + 2, columns + halo, 8 channels;
 //     zero fill outside the image is the padding) arrives by a tensor-map copy
 //     (per-thread loads when x is not 16-byte aligned or W % 4 != 0), and the
@@ -79,7 +82,10 @@ constexpr int NLOAD = 256;         // loader threads (warps 0-7)
 constexpr int MMA_WARP = 8;        // warp 8: TMEM owner and MMA issuer
 constexpr int EPI_WARP0 = 9;       // warps 9-16: epilogue, two per TMEM lane quadrant
 constexpr int NEPI = 256;          // epilogue threads
-constexpr int NTHREADS = 544;
+constexpr int WPROD_WARP = 17;     // warp 17: weight producer (weight-ring instantiations only)
+constexpr int NGRP = 3;            // weight-ring groups per chunk
+constexpr int TPG = NTAP / NGRP;   // taps per weight-ring group
+constexpr int WSL_MAX = 12;        // weight-ring slots at most (4 chunks)
 constexpr int LBATCH = 4;          // loader items whose global loads are in flight together
 constexpr long WAIT_LIMIT = PP_WAIT_POLLS;  // mbarrier polls before a wait gives up
 // dynamic shared memory a CTA may request: 227 KB less room for the kernel's static barriers
@@ -146,6 +152,18 @@ struct Geo {
   static constexpr int LO_BYTES = IN_BYTES > RAW ? IN_BYTES : RAW;
   static constexpr int W_TILE = FB * KC * 4;              // one tap, one of hi / lo (FB x 8 fp32 or FB x 16 f16)
   static constexpr int W_BYTES = NTAP * 2 * W_TILE;       // weights of one chunk
+  // WR: the weights sit in a ring of WSL groups of TPG taps (GRP bytes each, two
+  // chunks at least, up to WSL_MAX as shared memory allows) ahead of the two
+  // input operand stages, filled by the producer warp; a group's slot is
+  // refilled as soon as its MMAs complete.  Used by the tf32 128-filter tiles,
+  // where it measured faster; the others (the 64-filter tiles are shared-memory
+  // bound at 9 taps of N = 128 + 64 MMAs) keep each chunk's weights in its
+  // operand stage, copied whole by the loaders' thread 0 once the stage is free,
+  // and run without the producer warp (an 18th warp, even idle, measured slower
+  // there).
+  static constexpr bool WR = FB == 128 && !F16;
+  static constexpr int NTHREADS = WR ? 576 : 544;
+  static constexpr int GRP = W_BYTES / NGRP;
   // SEP: the raw boxes get a ring of their own (NRAW = two slots, or one when
   // two do not fit), so the copy for chunk g + NRAW starts as soon as chunk g's
   // box has been read instead of waiting for the MMAs that read the stage; used
@@ -155,13 +173,18 @@ struct Geo {
   static constexpr int NRAW = 2 * STAGE_SEP + 2 * RAW + 1024 <= SMEM_LIMIT ? 2
                               : (2 * STAGE_SEP + RAW + 1024 <= SMEM_LIMIT ? 1 : 0);
   static constexpr bool SEP = NRAW > 0;
-  static constexpr int STAGE = SEP ? STAGE_SEP : W_BYTES + IN_BYTES + LO_BYTES;
-  static constexpr int RAW_OFF = 2 * STAGE;               // raw slots (SEP)
-  static constexpr int SMEM_ALLOC = 2 * STAGE + NRAW * RAW + 1024;
+  static constexpr int XSTAGE = SEP ? 2 * IN_BYTES : IN_BYTES + LO_BYTES;  // input operands (hi, lo) of a stage
+  static constexpr int STAGE = WR ? XSTAGE : W_BYTES + XSTAGE;  // stage stride; without WR its weights come first
+  static constexpr int WSL_FIT = (SMEM_LIMIT - 1024 - 2 * XSTAGE - NRAW * RAW) / GRP;
+  static constexpr int WSL = WR ? (WSL_FIT < WSL_MAX ? WSL_FIT : WSL_MAX) : 0;
+  static constexpr int XOFF = WR ? WSL * GRP : W_BYTES;  // stage s's input operands at XOFF + s * STAGE
+  static constexpr int RAW_OFF = WR ? XOFF + 2 * STAGE : 2 * STAGE;  // raw slots (SEP)
+  static constexpr int SMEM_ALLOC = RAW_OFF + NRAW * RAW + 1024;
   static constexpr int ITEMS = (2 * NPIX + NLOAD - 1) / NLOAD;  // (K half, pixel) items per loader thread
   static_assert(SMEM_ALLOC <= SMEM_LIMIT, "shared memory plan");
-  static_assert(W_BYTES % 128 == 0 && IN_BYTES % 128 == 0 && RAW % 128 == 0 && STAGE % 128 == 0,
+  static_assert(W_BYTES % 128 == 0 && IN_BYTES % 128 == 0 && RAW % 128 == 0 && STAGE % 128 == 0 && GRP % 128 == 0,
                 "tensor-map copies need 128-byte aligned shared-memory destinations");
+  static_assert(!WR || WSL >= 2 * NGRP, "the weight ring holds two chunks at least");
   static constexpr uint32_t IDESC = F16 ? (ORI == ORI_FP ? idesc_f16(128, TW) : idesc_f16(128, FB))
                                         : (ORI == ORI_FP ? idesc_tf32(128, TW) : idesc_tf32(128, FB));
   static constexpr uint32_t IDESC2 = F16 ? idesc_f16(128, 2 * FB) : idesc_tf32(128, 2 * FB);  // MRG: [w_hi | w_lo]
@@ -185,7 +208,7 @@ __device__ __forceinline__ Tile tile_of(const TcParams& p, int t, int R, int TW)
 }
 
 template <int ORI, int TW, int FB, bool F16>
-__global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p, const __grid_constant__ CUtensorMap xmap) {
+__global__ void __launch_bounds__(Geo<ORI, TW, FB, F16>::NTHREADS, 1) ppconv_tc_kernel(const TcParams p, const __grid_constant__ CUtensorMap xmap) {
   using G = Geo<ORI, TW, FB, F16>;
   // slots of the box ring (its uses sit behind G::SEP; 1 keeps the modulo defined where the ring is absent)
   constexpr int RING = G::NRAW > 0 ? G::NRAW : 1;
@@ -194,6 +217,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
   // compiler keeps every access below in the shared state space.
   unsigned char* smem = smem_raw + ((1024u - (su32(smem_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t full[2], empty[2], acc_full[2], acc_empty[2], done_bar, raw_full[2];
+  __shared__ __align__(8) uint64_t wempty[G::WR ? WSL_MAX : 1];  // a weight-ring slot has been read by its MMAs
   __shared__ uint32_t tmem_s;
   __shared__ volatile int abort_s;
 
@@ -213,15 +237,18 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
-      // full: every loader thread's operand stores plus the weight copy (one
-      // more arrival, with its bytes), so the MMA thread waits once per chunk
-      mbar_init(su32(&full[s]), NLOAD + 1);
+      // full: every loader thread's operand stores plus the chunk's weight
+      // copies (one more arrival each, with its bytes: the whole chunk, or its
+      // NGRP ring groups), so the MMA thread waits once per chunk
+      mbar_init(su32(&full[s]), NLOAD + (G::WR ? NGRP : 1));
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
       mbar_init(su32(&acc_empty[s]), NEPI);
       mbar_init(su32(&raw_full[s]), 1);
     }
     mbar_init(su32(&done_bar), 1);
+    if (G::WR)
+      for (int k = 0; k < WSL_MAX; ++k) mbar_init(su32(&wempty[k]), 1);
     abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -238,9 +265,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
 
   if (warp < MMA_WARP) {
     // ------------------------------------------------------------ loaders
-    // Thread 0 issues the copies: weights (bulk, on full[s]) and, with a tensor
-    // map, the raw input box (on raw_full); all loader threads then transpose the
-    // box into the hi / lo operand tiles and arrive on full[s].
+    // Thread 0 issues the copies: the weights (bulk, on full[s]) unless the
+    // producer warp does (WR) and, with a tensor map, the raw input box (on
+    // raw_full); all loader threads then transpose the box into the hi / lo
+    // operand tiles and arrive on full[s].
     const int nall = nmine * p.nch;  // chunks of this CTA
     auto issue_raw = [&](int gg, unsigned char* dst) {  // thread 0 only
       const int i = gg / p.nch, c = gg - i * p.nch;
@@ -270,7 +298,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
     // The weights do not depend on the previous kernel in the stream: the first
     // two chunks' copies start before waiting for it (programmatic dependent
     // launch), everything that reads x comes after the wait.
-    if (tid == 0)
+    if (!G::WR && tid == 0)
       for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && G::SEP)
@@ -284,12 +312,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       const float* xb = p.x + (size_t)T.n * p.Ci * p.H * p.W;
       for (int c = 0; c < p.nch; ++c, ++g) {
         const int s = g & 1, use = g >> 1;
-        // f16 with a box ring: the box of this chunk has a slot of its own and lands ahead of time, so it is
-        // read and split into registers before the stage is free (while the MMAs of the two previous chunks
-        // still read it); only the stores wait for the stage.
-        constexpr int EI = (F16 && G::SEP) ? G::ITEMS : 1;
+        // f16 (and the tf32 weight-ring tiles) with a box ring: the box of this chunk has a slot of its own and
+        // lands ahead of time, so it is read and split into registers before the stage is free (while the
+        // MMAs of the two previous chunks still read it); only the stores wait for the stage.
+        constexpr bool EARLY = (F16 || G::WR) && G::SEP;
+        constexpr int EI = EARLY ? G::ITEMS : 1;
         uint4 hreg[EI], lreg[EI];
-        const bool early = F16 && G::SEP && p.use_tma;
+        const bool early = EARLY && p.use_tma;
         if (early) {
           if (group_any<NLOAD>(!wait(&raw_full[g & 1], (uint32_t)((g >> 1) & 1)))) {
             stop = true;
@@ -306,7 +335,19 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
               float u[G::CPH];
 #pragma unroll
               for (int k = 0; k < G::CPH; ++k) u[k] = raw[((kh * G::CPH + k) * G::BROWS + br) * G::RAW_W + bc + 3];
-              range_bad |= split_f16x8(u, p.xscale, hreg[b], lreg[b]);
+              if constexpr (F16) {
+                range_bad |= split_f16x8(u, p.xscale, hreg[b], lreg[b]);
+              } else {
+                // tf32 split: hi keeps the top 10 mantissa bits (exact in tf32), lo = v - hi (exact in fp32)
+                uint32_t hb[4], lb[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  hb[k] = __float_as_uint(u[k]) & 0xFFFFE000u;
+                  lb[k] = __float_as_uint(u[k] - __uint_as_float(hb[k]));
+                }
+                hreg[b] = make_uint4(hb[0], hb[1], hb[2], hb[3]);
+                lreg[b] = make_uint4(lb[0], lb[1], lb[2], lb[3]);
+              }
             }
           }
           // the slot is rewritten next by a tensor-map copy: reads ordered before it, then released
@@ -321,11 +362,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
           stop = true;
           break;
         }
-        unsigned char* st = smem + s * G::STAGE;
-        float4* hi = reinterpret_cast<float4*>(st + G::W_BYTES);
-        float4* lo = reinterpret_cast<float4*>(st + G::W_BYTES + G::IN_BYTES);
+        unsigned char* st = smem + G::XOFF + s * G::STAGE;
+        float4* hi = reinterpret_cast<float4*>(st);
+        float4* lo = reinterpret_cast<float4*>(st + G::IN_BYTES);
         if (tid == 0) {
-          if (g >= 2) {
+          if (!G::WR && g >= 2) {
             issue_w(g, s);
             ++w_issued;
           }
@@ -458,7 +499,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
   } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      int g = 0;
+      int g = 0, wslot = 0;  // chunk count and (WR) the weight-ring slot of the next group
       for (int i = 0; i < nmine && !abort_s; ++i) {
         const int b = i & 1, ub = i >> 1;
         if (ub > 0 && !wait(&acc_empty[b], (uint32_t)((ub - 1) & 1))) break;
@@ -472,17 +513,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
             break;
           }
           tm_fence_after();
-          const unsigned char* st = smem + s * G::STAGE;
+          const unsigned char* st = smem + G::XOFF + s * G::STAGE;
           // Descriptors hold address / 16 in their low 14 bits and every operand
           // lies below 256 KB, so moving an operand is one add to the descriptor.
-          const uint64_t w0 = smem_desc(su32(st), G::WLBO);
-          const uint64_t xh0 = smem_desc(su32(st + G::W_BYTES), G::IN_HALF);
-          const uint64_t xl0 = smem_desc(su32(st + G::W_BYTES + G::IN_BYTES), G::IN_HALF);
+          const uint64_t w0 = smem_desc(su32(smem + s * G::STAGE), G::WLBO);  // without WR
+          const uint64_t xh0 = smem_desc(su32(st), G::IN_HALF);
+          const uint64_t xl0 = smem_desc(su32(st + G::IN_BYTES), G::IN_HALF);
+          int gs[NGRP];  // WR: the chunk's weight groups, consecutive slots of the ring
+#pragma unroll
+          for (int k = 0; k < NGRP; ++k) {
+            gs[k] = wslot;
+            if (G::WR) wslot = wslot + 1 == G::WSL ? 0 : wslot + 1;
+          }
           const uint32_t acc0 = c == 0 ? 0u : 1u;  // the tile's first chunk overwrites the accumulators
 #pragma unroll
           for (int t = 0; t < NTAP; ++t) {
             const int dy = t / 3, dx = t % 3;
-            const uint64_t whi = w0 + (uint64_t)((t * 2 + 0) * G::W_TILE / 16);
+            const uint64_t whi = G::WR ? smem_desc(su32(smem + gs[t / TPG] * G::GRP + (t % TPG) * 2 * G::W_TILE), G::WLBO)
+                                       : w0 + (uint64_t)(t * 2 * G::W_TILE / 16);
             const uint64_t wlo = whi + (uint64_t)FB;  // lo rows follow the hi rows: FB rows of 16 bytes
 #pragma unroll(G::NSEG <= 8 ? G::NSEG : 4)
             for (int rr = 0; rr < G::NSEG; ++rr) {
@@ -512,6 +560,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
                 mma_tf32(d, xl, whi, G::IDESC, 1u);
               }
             }
+            if (G::WR && t % TPG == TPG - 1) mma_commit(su32(&wempty[gs[t / TPG]]));  // slot free once these complete
           }
           mma_commit(su32(&empty[s]));
         }
@@ -524,6 +573,47 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tc_kernel(const TcParams p
       asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
       mma_commit(su32(&done_bar));
       wait(&done_bar, 0u);
+    }
+    __syncwarp();
+  } else if (warp == WPROD_WARP) {
+    // ------------------------------------------------------------ weight producer (WR)
+    // A chunk's weights are NGRP groups of TPG tap tiles, copied into the ring of
+    // G::WSL slots.  A group is copied as soon as the MMAs of the group that held
+    // its slot before have completed; the chunk's copies arrive (with their bytes)
+    // on the stage's full barrier, and those of chunk g go out only after that
+    // barrier's previous phase (chunk g - 2) has completed.
+    if (G::WR && lane == 0) {
+      const int nall = nmine * p.nch;
+      int slot = 0, use = 0, issued = 0;  // ring position, its round, groups issued
+      bool ok = true;
+      for (int gg = 0; gg < nall && ok; ++gg) {
+        const int s = gg & 1;
+        if (gg >= 2) ok = wait(&full[s], (uint32_t)(((gg - 2) >> 1) & 1));
+        const Tile T = tile_of(p, (int)blockIdx.x + (gg / p.nch) * (int)gridDim.x, G::R, TW);
+        const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + gg % p.nch) * G::W_BYTES;
+        for (int k = 0; k < NGRP && ok; ++k) {
+          if (use > 0) ok = wait(&wempty[slot], (uint32_t)((use - 1) & 1));
+          if (!ok) break;
+          mbar_arrive_expect_tx(su32(&full[s]), G::GRP);
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                  su32(smem + slot * G::GRP)),
+              "l"(src + (size_t)k * G::GRP), "r"(G::GRP), "r"(su32(&full[s]))
+              : "memory");
+          ++issued;
+          if (++slot == G::WSL) {
+            slot = 0;
+            ++use;
+          }
+        }
+      }
+      // No copy may still be writing shared memory when the CTA exits: wait
+      // (bounded) for the last two chunks' barriers (after a timeout a barrier
+      // may lack loader arrivals; the bounded wait outlasts any copy in flight).
+      const int last = (issued + NGRP - 1) / NGRP;
+      for (int gg = last > 2 ? last - 2 : 0; gg < last; ++gg)
+        for (long w = 0; w < WAIT_LIMIT && !mbar_try(su32(&full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++w) {
+        }
     }
     __syncwarp();
   } else {
@@ -788,7 +878,7 @@ cudaError_t launch_one(const TcParams& p0, cudaStream_t stream, int sms) {
   p.ntiles = (int)nt;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)std::min<int64_t>(nt, sms));
-  cfg.blockDim = dim3(NTHREADS);
+  cfg.blockDim = dim3(G::NTHREADS);
   cfg.dynamicSmemBytes = G::SMEM_ALLOC;
   cfg.stream = stream;
   // programmatic dependent launch: the kernel waits (griddepcontrol.wait) for
