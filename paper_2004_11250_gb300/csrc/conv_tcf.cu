@@ -76,8 +76,8 @@ constexpr int NLOAD = 256;            // loader threads (warps 0-7)
 constexpr int MMA_WARP = 8;
 constexpr int EPI_WARP0 = 9;          // warps 9-16
 constexpr int NEPI = 256;
-constexpr int WPROD_WARP = 17;        // the weight producer
-constexpr int NTHREADS = 576;
+constexpr int WPROD_WARP = 17;        // the weight producer (weight-ring instantiations)
+constexpr int NTHREADS = 576;         // with the producer warp; 544 without
 constexpr int WMAX = 128;             // widest map handled
 constexpr int W_TILE = FB * KC * 4;   // one tap, hi or lo: 128 x 8 fp32 (or 128 x 16 f16)
 constexpr int TAP_BYTES = 2 * W_TILE;          // one tap's hi and lo rows
@@ -95,6 +95,16 @@ constexpr int MAX_SPLIT = 16;
 static_assert(2 * (W_BYTES + 2 * IN_MAX) <= SMEM_USE, "shared memory plan");
 static_assert(GRP_BYTES % 1024 == 0, "weight-ring slots keep 1024-byte alignment");
 static_assert(FB * NMAX * 4 <= SMEM_USE, "split reduction buffer");
+
+// Weights by the producer warp into the ring of 3-tap groups: the cluster-split
+// and f16 instantiations.  The unsplit tf32 one (persistent over several tiles)
+// measured faster with each chunk's weights copied whole by the loaders' thread
+// 0 into two fixed chunk slots (the ring's first 6 group slots) once the stage
+// is free, and without the producer warp (an 18th warp, even idle, slowed it).
+template <bool SPLIT, bool F16>
+__host__ __device__ constexpr bool weight_ring() { return SPLIT || F16; }
+template <bool SPLIT, bool F16>
+__host__ __device__ constexpr int flat_threads() { return weight_ring<SPLIT, F16>() ? NTHREADS : NTHREADS - 32; }
 
 struct FlatParams {
   const float* rscale;      // f16: per reordered filter, 1 / (weight scale x input scale)
@@ -237,8 +247,9 @@ __device__ __forceinline__ void split_reduce(const FlatParams& p, const Tile& T,
 // reported its stage full, and its commits arrive in both CTAs.  Pairs run in
 // cluster-split mode (one tile per CTA).
 template <bool SPLIT, bool F16, bool PAIR>
-__global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
+__global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kernel(const FlatParams p, const __grid_constant__ CUtensorMap xmap) {
   static_assert(SPLIT || !PAIR, "CTA pairs run in cluster-split mode");
+  constexpr bool WR = weight_ring<SPLIT, F16>();
   constexpr int KCH = F16 ? 16 : KC;  // input channels per chunk
   constexpr int CPH = KCH / 2;         // channels per K half (16 bytes of one pixel row of an operand)
   extern __shared__ unsigned char smem_raw[];
@@ -269,17 +280,18 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
   if (tid == 0) {
     for (int s = 0; s < 2; ++s) {
       // a stage is full once every loader thread has stored its part of the
-      // input operands and the chunk's three weight-group copies (three more
-      // arrivals, with their bytes) have landed: the MMA thread waits on one
-      // barrier per chunk
-      mbar_init(su32(&full[s]), NLOAD + NGRP);
+      // input operands and the chunk's weight copies (one more arrival each,
+      // with its bytes: the three group copies, or without the ring the whole
+      // chunk) have landed: the MMA thread waits on one barrier per chunk
+      mbar_init(su32(&full[s]), NLOAD + (WR ? NGRP : 1));
       mbar_init(su32(&raw_full[s]), 1);
       mbar_init(su32(&empty[s]), 1);
       mbar_init(su32(&acc_full[s]), 1);
       mbar_init(su32(&acc_empty[s]), NEPI);
     }
     mbar_init(su32(&done_bar), 1);
-    for (int k = 0; k < WSL_MAX; ++k) mbar_init(su32(&wempty[k]), 1);
+    if (WR)
+      for (int k = 0; k < WSL_MAX; ++k) mbar_init(su32(&wempty[k]), 1);
     mbar_init(su32(&pfull[0]), 1);
     mbar_init(su32(&pfull[1]), 1);
     abort_s = 0;
@@ -386,9 +398,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     };
     // With a ring of their own the boxes are copied one or two chunks ahead of use
     // (as many as the ring has slots), not only once the chunk's stage is free.
-    int g = 0, raw_issued = 0;
-    // Everything that reads x comes after the wait for the previous kernel in
-    // the stream (programmatic dependent launch).
+    int g = 0, raw_issued = 0, w_issued = 0;
+    // Without the ring: the weights of chunk gg, whole, into chunk slot s (the
+    // ring's group slots 3 s .. 3 s + 2), on the stage's full barrier (thread 0).
+    auto issue_w = [&](int gg, int s) {
+      const Tile T = my_tile(tile_index(gg / nchm));
+      const unsigned char* src = p.wt + ((size_t)T.fb * p.nch + c_beg + gg % nchm) * W_BYTES;
+      mbar_arrive_expect_tx(su32(&full[s]), W_BYTES);
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              su32(smem + (size_t)s * W_BYTES)),
+          "l"(src), "r"(W_BYTES), "r"(su32(&full[s]))
+          : "memory");
+    };
+    // The weights do not depend on the previous kernel in the stream: without
+    // the ring the first two chunks' copies start before waiting for it
+    // (programmatic dependent launch); everything that reads x comes after.
+    if (!WR && tid == 0)
+      for (; w_issued < 2 && w_issued < nall; ++w_issued) issue_w(w_issued, w_issued);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (tid == 0 && p.use_tma && p.sep)
       for (; raw_issued < p.sep && raw_issued < nall; ++raw_issued)
@@ -469,6 +496,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
         float4* hi = reinterpret_cast<float4*>(st);
         float4* lo = reinterpret_cast<float4*>(st + p.lo_off);
         if (tid == 0) {
+          if (!WR && g >= 2) {
+            issue_w(g, s);
+            ++w_issued;
+          }
           if (p.use_tma && !p.sep) {
             issue_raw(g, reinterpret_cast<unsigned char*>(lo));  // lands in the lo operand, split in place below
             ++raw_issued;
@@ -533,6 +564,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
       // bounded wait then outlasts any copy still in flight.)
       for (int gg = raw_issued > 2 ? raw_issued - 2 : 0; gg < raw_issued; ++gg)
         for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&raw_full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
+        }
+      for (int gg = w_issued > 2 ? w_issued - 2 : 0; gg < w_issued; ++gg)
+        for (long k = 0; k < WAIT_LIMIT && !mbar_try(su32(&full[gg & 1]), (uint32_t)((gg >> 1) & 1)); ++k) {
         }
     }
     __syncwarp();
@@ -603,7 +637,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
               mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
               mma_tf32(d, whi, xl0 + off, p.idesc, 1u);
             }
-            if (t % 3 == 2) {  // the group's slot is free for the producer once these MMAs complete
+            if (WR && t % 3 == 2) {  // the group's slot is free for the producer once these MMAs complete
               if (PAIR)
                 mma_commit_pair(su32(&wempty[gs[t / 3]]), pmask);
               else
@@ -642,7 +676,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) ppconv_tcf_kernel(const FlatParam
     // arrive (with their bytes) on the stage's full barrier, so the MMA thread
     // still waits once per chunk; the copies of chunk g go out only after the
     // barrier's previous phase (chunk g - 2) has completed.
-    if (lane == 0) {
+    if (WR && lane == 0) {
       const int nchm = c_end - c_beg;
       const int nall = nmine * nchm;
       int slot = 0, use = 0, issued = 0;  // ring position, its round, groups issued
@@ -1125,12 +1159,14 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.npixa = G.npixa;
   p.raw_w = G.raw_w;
   p.raw_bytes = G.raw_bytes;
-  p.wsl = G.wsl;
-  p.xoff = G.xoff;
+  // without the weight ring (unsplit tf32): two whole-chunk weight slots, 6 group slots
+  const bool ring = G.split > 1 || G.pair || f16;
+  p.wsl = ring ? G.wsl : 6;
+  p.xoff = p.wsl * GRP_BYTES;
   p.xstage = G.xstage;
   p.lo_off = G.lo_off;
   p.sep = G.sep;
-  p.raw_off = G.raw_off;
+  p.raw_off = p.xoff + 2 * G.xstage;
   p.raw_slot = G.raw_slot;
   p.tiles_y = G.tiles_y;
   p.ntiles = G.ntiles;
@@ -1181,7 +1217,7 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  cfg.blockDim = dim3(NTHREADS);
+  cfg.blockDim = dim3(ring ? flat_threads<true, false>() : flat_threads<false, false>());
   cfg.dynamicSmemBytes = SMEM_ALLOC;
   cfg.stream = stream;
   cudaError_t e;
