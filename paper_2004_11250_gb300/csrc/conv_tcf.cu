@@ -43,11 +43,15 @@
 // scaling (|x s| >= 65520) or are not finite are flagged by the loaders in the
 // device status word.
 //
-// Roles (17 warps, one CTA per SM): warps 0-7 stage the operands (thread 0
-// also issues the weight and input-box copies), warp 8 allocates TMEM and one
-// of its threads issues the MMAs, waiting once per chunk (the stage's full
-// barrier counts the loaders and the weight copy), warps 9-16 are the
-// epilogue (two per TMEM lane quadrant).  Without a split the CTA is persistent
+// Roles (one CTA per SM): warps 0-7 stage the operands (thread 0 also issues
+// the input-box copies), warp 8 allocates TMEM and one of its threads issues
+// the MMAs, waiting once per chunk (the stage's full barrier counts the loaders
+// and the weight copies), warps 9-16 are the epilogue (two per TMEM lane
+// quadrant), and in the cluster-split and f16 instantiations warp 17 copies
+// the weights, three groups of 3 taps per chunk into a ring of group slots,
+// each slot refilled as soon as its MMAs complete.  The unsplit tf32
+// instantiation has no warp 17: loader thread 0 copies each chunk's weights
+// whole once its stage is free.  Without a split the CTA is persistent
 // over tiles with two TMEM accumulator buffers, so a tile's epilogue overlaps
 // the next tile's MMAs.  Every mbarrier wait is bounded; a timeout sets the
 // layer's device status word and the CTA skips the rest of its work (every
@@ -948,7 +952,7 @@ cudaError_t init_device(int dev) {
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    // both precisions launch 544 threads, one CTA per SM, with the same shared memory
+    // split launches run 576 threads in both precisions, one CTA per SM, with the same shared memory
     if (cudaOccupancyMaxActiveClusters(&n, ppconv_tcf_kernel<true, false, false>, &cfg) != cudaSuccess) {
       cudaGetLastError();
       n = 0;
