@@ -37,7 +37,8 @@
 // layer by powers of two so that both stay in fp16's normal range; a chunk is
 // 16 channels (the K of kind::f16) and each tap runs w_hi x_hi into one
 // accumulator and w_lo x_hi + w_hi x_lo into a second one (TMEM columns 128 ..
-// 255 of the buffer), combined in the epilogue as (acc1 + 2^-11 acc2) times the
+// 255 of the buffer for tiles of at most 128 columns; for wider tiles, which run
+// one per CTA, the other buffer), combined in the epilogue as (acc1 + 2^-11 acc2) times the
 // filter's inverse scale.  The dropped lo x lo term and the rounding of the lo
 // parts are each below 2^-22 of |w * x|.  Inputs that overflow fp16 after
 // scaling (|x s| >= 65520) or are not finite are flagged by the loaders in the
@@ -72,7 +73,7 @@ namespace {
 using namespace ppc_ptx;
 
 constexpr int KC = 8;                 // input channels per chunk (MMA K for tf32; 16 for f16)
-constexpr int ACC2 = 128;             // f16: column offset of the second accumulator in a buffer
+constexpr int ACC2 = 128;             // f16, double-buffered: column offset of the second accumulator in a buffer
 constexpr int NTAP = 9;
 constexpr int FB = 128;               // filters per block (MMA M)
 constexpr int NMAX = 256;             // TMEM columns of one accumulator buffer
@@ -130,6 +131,10 @@ struct FlatParams {
   int plane;                // box over x viewed as [N][Ci][H * W]: the staged rows packed, raw_w = box width
   int tiles_y, ntiles, split;
   uint32_t idesc;
+  // TMEM accumulator buffers (2: a tile's epilogue overlaps the next tile's MMAs;
+  // 1: f16 tiles wider than ACC2 columns, whose second accumulator takes the
+  // other buffer's columns) and the f16 second accumulator's column offset
+  int nbuf, acc2;
 };
 
 struct Tile {
@@ -590,10 +595,11 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
     } else if (lane == 0) {
       int g = 0, wslot = 0;  // chunk count and the weight-ring slot of the next group
       for (int i = 0; i < nmine && !abort_s; ++i) {
-        const int b = i & 1, ub = i >> 1;
+        const int b = p.nbuf == 2 ? (i & 1) : 0, ub = p.nbuf == 2 ? (i >> 1) : i;
         if (ub > 0 && !wait(&acc_empty[b], (uint32_t)((ub - 1) & 1))) break;
         tm_fence_after();
         const uint32_t d = tmem + (uint32_t)(b * NMAX);
+        const uint32_t d2 = d + (uint32_t)p.acc2;  // f16: the second accumulator
         bool okc = true;
         for (int c = c_beg; c < c_end; ++c, ++g) {
           const int s = g & 1, use = g >> 1;
@@ -624,8 +630,8 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
             if (PAIR) {
               if (F16) {
                 mma_f16_pair(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
-                mma_f16_pair(d + ACC2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
-                mma_f16_pair(d + ACC2, whi, xl0 + off, p.idesc, 1u);
+                mma_f16_pair(d2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+                mma_f16_pair(d2, whi, xl0 + off, p.idesc, 1u);
               } else {
                 mma_tf32_pair(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
                 mma_tf32_pair(d, wlo, xh0 + off, p.idesc, 1u);
@@ -634,8 +640,8 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
             } else if (F16) {
               // acc1 += w_hi x_hi; acc2 += w_lo x_hi + w_hi x_lo (both lo parts scaled by 2^11)
               mma_f16(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
-              mma_f16(d + ACC2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
-              mma_f16(d + ACC2, whi, xl0 + off, p.idesc, 1u);
+              mma_f16(d2, wlo, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
+              mma_f16(d2, whi, xl0 + off, p.idesc, 1u);
             } else {
               mma_tf32(d, whi, xh0 + off, p.idesc, t == 0 ? acc0 : 1u);
               mma_tf32(d, wlo, xh0 + off, p.idesc, 1u);
@@ -723,12 +729,13 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
     const bool relu = p.flags & PP_RELU;
     const float* skip = (p.flags & PP_ADD_SKIP) ? p.skip : nullptr;
     for (int i = 0; i < nmine; ++i) {
-      const int b = i & 1, ub = i >> 1;
+      const int b = p.nbuf == 2 ? (i & 1) : 0, ub = p.nbuf == 2 ? (i >> 1) : i;
       // the whole warp leaves together: its TMEM loads are warp-collective
       if (!__all_sync(0xffffffffu, wait(&acc_full[b], (uint32_t)(ub & 1)))) break;
       tm_fence_after();
       const Tile T = my_tile(tile_index(i));
       const uint32_t lanebase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * NMAX);
+      const uint32_t lane2 = lanebase + (uint32_t)p.acc2;  // f16: the second accumulator
       const int m = 32 * q + lane;  // filter within the block = TMEM lane
       // f16: the filter's inverse scale (the layout holds nfb x FB entries, padding included)
       const float rs = F16 ? __ldg(p.rscale + T.fb * FB + m) : 1.f;
@@ -745,7 +752,7 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
           for (int u = 0; u < 4; ++u)
             if (cb0 + 16 * u < p.ncols) {
               tm_ld8(lanebase + (uint32_t)(cb0 + 16 * u), a[u]);
-              if constexpr (F16) tm_ld8(lanebase + (uint32_t)(ACC2 + cb0 + 16 * u), a2[u]);
+              if constexpr (F16) tm_ld8(lane2 + (uint32_t)(cb0 + 16 * u), a2[u]);
             }
           tm_wait_ld();
           if constexpr (F16) {
@@ -779,7 +786,7 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
             for (int cb = 0; cb < p.W; cb += 8) {
               float a[8], a2[8];
               tm_ld8(lanebase + (uint32_t)(rr * p.bcols + cb), a);
-              if constexpr (F16) tm_ld8(lanebase + (uint32_t)(ACC2 + rr * p.bcols + cb), a2);
+              if constexpr (F16) tm_ld8(lane2 + (uint32_t)(rr * p.bcols + cb), a2);
               tm_wait_ld();
               if constexpr (F16) {
 #pragma unroll
@@ -815,8 +822,8 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
               tm_ld8(lanebase + (uint32_t)(rr * p.bcols + cb), a);
               tm_ld8(lanebase + (uint32_t)((rr + 1) * p.bcols + cb), bb);
               if constexpr (F16) {
-                tm_ld8(lanebase + (uint32_t)(ACC2 + rr * p.bcols + cb), a2);
-                tm_ld8(lanebase + (uint32_t)(ACC2 + (rr + 1) * p.bcols + cb), bb2);
+                tm_ld8(lane2 + (uint32_t)(rr * p.bcols + cb), a2);
+                tm_ld8(lane2 + (uint32_t)((rr + 1) * p.bcols + cb), bb2);
               }
               tm_wait_ld();
               if constexpr (F16) {
@@ -996,13 +1003,15 @@ struct FlatGeo {
 // cycle; and clusters beyond those co-resident on the GPU run in later waves.
 // Every geometry the kernel can run for this shape, best first by the model;
 // fills up to maxn entries and returns how many.
-// f16: nch counts 16-channel chunks, an accumulator is at most 128 columns (the
-// second one follows it in the same buffer) and the input box holds 16 channels.
+// f16: nch counts 16-channel chunks and the input box holds 16 channels; a tile
+// of at most 128 columns keeps its second accumulator in the same TMEM buffer
+// (double-buffered), a wider one puts it in the other buffer (single-buffered:
+// only where each CTA has one tile).
 int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
                     FlatGeo* out, int maxn, bool f16) {
   if (W < 1 || W > WMAX || H < 1 || maxn < 1) return 0;
   const int bcols = (W + 2 + 7) / 8 * 8;
-  const int nmax = f16 ? ACC2 : NMAX;
+  const int nmax = NMAX;  // f16 tiles wider than ACC2 run single-buffered (below)
   const int kch = f16 ? 16 : KC;
   const int rmax = nmax / bcols;
   if (rmax < 1 || (pool && rmax < 2)) return 0;
@@ -1046,6 +1055,11 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
       G.xoff = G.wsl * GRP_BYTES;
       G.raw_off = G.xoff + 2 * G.xstage;
       if (G.npixa > PIX_MAX || !fits(G.wsl, G.sep) || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
+      // f16 with more than ACC2 columns: the second accumulator takes the other TMEM buffer, so the
+      // tile is single-buffered; allowed where each CTA has one tile (cluster split, or an unsplit grid
+      // of at most one tile per SM), and not for pairs
+      const bool wide = f16 && G.ncols > ACC2;
+      if (wide && pair) continue;
       G.ntiles = (int)nt;
       const double mma = 27.0 * std::max(G.ncols * 128.0 * 8.0 / 1850.0, 32.0 + G.ncols / 4.0);
       // pairs: each SM reads half the input operand bytes per MMA and issues half the MMAs; modelled as 0.8
@@ -1056,6 +1070,7 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
         const int cs = pair ? 2 * s : s;  // cluster size
         if (cs > MAX_SPLIT) break;
         if (cs > 1 && (!allow_split || s > nch || D.max_clusters[cs] <= 0 || (int64_t)G.ntiles * cs > D.sms)) continue;
+        if (cs == 1 && wide && G.ntiles > D.sms) continue;
         double cost;
         if (cs == 1) {
           const double waves = std::ceil((double)G.ntiles / D.sms);
@@ -1175,6 +1190,9 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.tiles_y = G.tiles_y;
   p.ntiles = G.ntiles;
   p.split = G.split;
+  const bool wide = f16 && G.ncols > ACC2;  // single-buffered f16 tile (one per CTA)
+  p.nbuf = wide ? 1 : 2;
+  p.acc2 = wide ? NMAX : ACC2;
   const int mrows = G.pair ? 2 * FB : FB;  // pairs: one M = 256 MMA over both CTAs' filter blocks
   p.idesc = f16 ? idesc_f16(mrows, G.ncols) : idesc_tf32(mrows, G.ncols);
   CUtensorMap xmap;
