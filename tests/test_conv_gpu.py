@@ -891,6 +891,66 @@ def test_f16_flat_kernel(pp, runner, oracle_mod, case, flags):
     check_within(g, y, s, f"f16 flat {case} {flags}")
 
 
+WIDE_F16_CASES = [
+    # N, Ci, Co, H, W, flags, whether split geometries exist; flat-kernel f16 tiles of more than 128 columns
+    # (the second accumulator in the other TMEM buffer, single-buffered) need one tile per CTA
+    (8, 64, 100, 56, 56, "relu", False),           # unsplit: 152 or 112 tiles of 3 or 4 rows; ragged filter block
+    (1, 96, 200, 28, 28, "skip_pool_relu", True),  # 8 or 10 tiles of 8 or 6 rows, unsplit and split 2 / 4
+    (2, 40, 130, 20, 30, "skip_relu", True),       # ragged channel chunk and filter block, unsplit and split 2
+]
+
+
+@pytest.mark.parametrize("case", WIDE_F16_CASES)
+def test_f16_flat_wide_tiles(pp, runner, oracle_mod, case):
+    """Every f16 flat-kernel geometry wider than 128 columns the planner accepts, two launches each, against
+    the oracle on every output; unsplit ones only where the grid has at most one tile per SM."""
+    N, Ci, Co, H, W, flags, split = case
+    rng = np.random.default_rng(N * 1000 + Ci + W)
+    L = synth.small_random_layer(rng, Co, Ci, P=8, keep=0.4)
+    x = rng.uniform(-1, 1, (N, Ci, H, W)).astype(np.float32)
+    skip = rng.uniform(-1, 1, (N, Co, H, W)).astype(np.float32) if "skip" in flags else None
+    relu, pool = "relu" in flags, "pool" in flags
+    y, s = oracle_layer_full(oracle_mod, L, x, skip, relu, pool)
+    f = (pp.PP_RELU if relu else 0) | (pp.PP_POOL2 if pool else 0) | (pp.PP_ADD_SKIP if skip is not None else 0)
+    Ho, Wo = (H // 2, W // 2) if pool else (H, W)
+    bcols = (W + 2 + 7) // 8 * 8
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    dl = runner.DeviceLayer(L, precision=F16)
+    try:
+        pp.pp_layer_set_kernel(dl.handle, pp.PP_KERNEL_TC_FLAT)
+        wide = []
+        for R in range(1, 17):
+            if (R * bcols + 15) // 16 * 16 <= 128:
+                continue
+            for S in (1, 2, 4, 8, 16):
+                try:
+                    pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, f, R, S)
+                except pp.PPError as e:
+                    assert e.code == pp.PP_ERR_UNSUPPORTED
+                    continue
+                tiles = -(-H // R) * -(-Co // 128) * N
+                if S == 1:
+                    assert tiles <= sms, (R, tiles)  # single-buffered: one tile per CTA
+                for rep in range(2):
+                    out = torch.full((N, Co, Ho, Wo), float("nan"), device="cuda")
+                    dl.forward(dev(x), out, None if skip is None else dev(skip), N, H, W, f,
+                               torch.cuda.current_stream())
+                    torch.cuda.synchronize()
+                    assert pp.pp_layer_device_status(dl.handle) == 0
+                    check_within(out.cpu().numpy(), y, s, f"{case} wide f16 R={R} S={S} #{rep}")
+                wide.append((R, S))
+        assert any(S == 1 for _, S in wide), wide
+        assert any(S > 1 for _, S in wide) == split, wide
+        # CTA pairs keep f16 tiles within 128 columns
+        for R in range(1, 17):
+            if (R * bcols + 15) // 16 * 16 > 128:
+                for S in (2, 4, 8):
+                    with pytest.raises(pp.PPError):
+                        pp.pp_layer_pin_flat_geometry(dl.handle, N, H, W, f, R, pp.PP_FLAT_PAIRED | S)
+    finally:
+        dl.close()
+
+
 @pytest.mark.parametrize("shape", [(1, 40, 130, 7, 100), (2, 16, 200, 4, 144), (1, 24, 64, 6, 160)] + PFR_CASES)
 @pytest.mark.parametrize("flags", ["none", "skip_relu", "pool_relu"])
 def test_f16_row_tiled(pp, runner, oracle_mod, shape, flags):
