@@ -439,12 +439,11 @@ __global__ void __launch_bounds__(flat_threads<SPLIT, F16>(), 1) ppconv_tcf_kern
         const int s = g & 1, use = g >> 1;
         // Without a tensor map the chunk's input values are fetched into
         // registers first: that needs no free stage, so it overlaps the wait.
-        // f16 with a box ring: the box has a slot of its own and lands ahead of
-        // time, so it is read and split into registers before the stage is free
-        // too, while the MMAs of the two previous chunks still read it (for tf32
-        // the split is cheap and waiting for the box first would only delay the
-        // chunk's weight copy, issued once the stage is free).
-        // v holds an item's input values, or (f16, split early) its packed hi words then lo words
+        // With a box ring the box has a slot of its own and lands ahead of time,
+        // so it is read into registers before the stage is free too, while the
+        // MMAs of the two previous chunks still read it; f16 also splits it
+        // there (the tf32 split is cheap and follows the stage wait).
+        // v holds an item's input values, or (f16, read early) its packed hi words then lo words
         float v[ITEMS_MAX][CPH];
         const bool early = p.use_tma && p.sep;
         if (early) {
