@@ -70,3 +70,41 @@ def test_roofline_time_is_the_slower_bound():
     assert bench.roof_time_s(peak, 0, 6756.2) == pytest.approx(1.0)
     assert bench.roof_time_s(0, 6756.2e9, 6756.2) == pytest.approx(1.0)
     assert bench.roof_time_s(peak, 2 * 6756.2e9, 6756.2) == pytest.approx(2.0)
+
+
+def test_source_hash_ignores_comments_only():
+    """The hash that ties profiles/ traffic figures to the kernel code skips // comments and blank lines,
+    and changes with any code edit."""
+    src = "int a = 1;  // one\n\n// a whole comment line\nint b = a + 2;\n"
+    assert bench.code_lines(src) == "int a = 1;\nint b = a + 2;"
+    assert bench.code_lines(src.replace("// one", "// another note")) == bench.code_lines(src)
+    assert bench.code_lines(src.replace("a + 2", "a + 3")) != bench.code_lines(src)
+
+
+def test_traffic_read_only_for_matching_code(tmp_path, monkeypatch):
+    """roofline.traffic comes from a committed summary only while that summary's recorded source hash is
+    the current one; otherwise the bench reports null."""
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "ppconv_vgg16_dram_traffic.txt").write_text(
+        "# summary\nkernel_source_sha256: abc\ndram_bytes_per_launch_avg: 1000\n"
+        "dram_bytes_per_launch_avg[ppconv_tcf_kernel]: 1234\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.traffic_from_profile("abc", "ppconv_tcf_kernel") == 1234.0
+    assert bench.traffic_from_profile("abc") == 1000.0
+    assert bench.traffic_from_profile("def", "ppconv_tcf_kernel") is None
+    assert bench.traffic_from_profile("abc", "ppconv_tcf_kernel", precision="f16x3") is None  # no such file
+
+
+def test_profile_commands_leave_clocks_alone():
+    """Every ncu command quoted in profiles/ runs with --clock-control none (ncu would otherwise lock
+    the GPU's clocks), and the summaries are short text."""
+    pdir = os.path.join(ROOT, "profiles")
+    names = sorted(os.listdir(pdir))
+    assert names
+    for name in names:
+        assert name.endswith((".md", ".txt")), name
+        text = open(os.path.join(pdir, name), encoding="utf-8").read()
+        assert len(text) < 16384, name
+        for line in text.splitlines():
+            if "ncu " in line and ("--metrics" in line or "--set" in line or "--section" in line):
+                assert "--clock-control none" in line, (name, line)
