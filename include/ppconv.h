@@ -302,8 +302,8 @@ pp_status pp_layer_autotune(pp_layer* layer, int N, int H, int W, int flags, voi
  * most 256 columns, R even when pooling; S a power of 2 up to 16, at most the
  * number of 8-channel chunks (16-channel in PP_PRECISION_F16X3), with tiles x S
  * within the SM count and the cluster size launchable on this GPU; in
- * PP_PRECISION_F16X3 a tile of more than 128 columns needs one tile per CTA:
- * S > 1, or at most one tile per SM, and no CTA pairs).  S | PP_FLAT_PAIRED names the same
+ * PP_PRECISION_F16X3 a tile of more than 128 columns runs single-buffered and
+ * not as CTA pairs).  S | PP_FLAT_PAIRED names the same
  * split run by CTA pairs: two filter blocks of a tile share each MMA (M = 256
  * over two SMs, cta_group::2), each SM staging half of the tile's pixels, in
  * clusters of 2 S CTAs (S up to 8; layers with an even number of 128-filter

@@ -37,8 +37,8 @@
 // layer by powers of two so that both stay in fp16's normal range; a chunk is
 // 16 channels (the K of kind::f16) and each tap runs w_hi x_hi into one
 // accumulator and w_lo x_hi + w_hi x_lo into a second one (TMEM columns 128 ..
-// 255 of the buffer for tiles of at most 128 columns; for wider tiles, which run
-// one per CTA, the other buffer), combined in the epilogue as (acc1 + 2^-11 acc2) times the
+// 255 of the buffer for tiles of at most 128 columns; for wider tiles, which are
+// single-buffered, the other buffer), combined in the epilogue as (acc1 + 2^-11 acc2) times the
 // filter's inverse scale.  The dropped lo x lo term and the rounding of the lo
 // parts are each below 2^-22 of |w * x|.  Inputs that overflow fp16 after
 // scaling (|x s| >= 65520) or are not finite are flagged by the loaders in the
@@ -1005,7 +1005,7 @@ struct FlatGeo {
 // f16: nch counts 16-channel chunks and the input box holds 16 channels; a tile
 // of at most 128 columns keeps its second accumulator in the same TMEM buffer
 // (double-buffered), a wider one puts it in the other buffer (single-buffered:
-// only where each CTA has one tile).
+// its epilogue is not overlapped with the CTA's next tile).
 int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow_split, const DeviceState& D,
                     FlatGeo* out, int maxn, bool f16) {
   if (W < 1 || W > WMAX || H < 1 || maxn < 1) return 0;
@@ -1055,8 +1055,8 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
       G.raw_off = G.xoff + 2 * G.xstage;
       if (G.npixa > PIX_MAX || !fits(G.wsl, G.sep) || G.ncols > nmax || nt > INT32_MAX / MAX_SPLIT) continue;
       // f16 with more than ACC2 columns: the second accumulator takes the other TMEM buffer, so the
-      // tile is single-buffered; allowed where each CTA has one tile (cluster split, or an unsplit grid
-      // of at most one tile per SM), and not for pairs
+      // tile is single-buffered (a CTA's next tile starts its MMAs once this one's epilogue has read
+      // the accumulators); not for pairs
       const bool wide = f16 && G.ncols > ACC2;
       if (wide && pair) continue;
       G.ntiles = (int)nt;
@@ -1069,11 +1069,11 @@ int flat_candidates(int N, int H, int W, int nch, int nfb, bool pool, bool allow
         const int cs = pair ? 2 * s : s;  // cluster size
         if (cs > MAX_SPLIT) break;
         if (cs > 1 && (!allow_split || s > nch || D.max_clusters[cs] <= 0 || (int64_t)G.ntiles * cs > D.sms)) continue;
-        if (cs == 1 && wide && G.ntiles > D.sms) continue;
         double cost;
         if (cs == 1) {
           const double waves = std::ceil((double)G.ntiles / D.sms);
-          cost = waves * nch * per_chunk + 5000.0;
+          // single-buffered: every tile's epilogue but the last is no longer hidden behind MMAs
+          cost = waves * nch * per_chunk + 5000.0 + (wide ? (waves - 1) * 16.0 * G.ncols : 0.0);
         } else {
           // clusters beyond those that fit on the GPU at once run in a later wave
           const double waves = std::ceil((double)G.ntiles / D.max_clusters[cs]);
@@ -1189,7 +1189,7 @@ pp_status launch_geo(const FlatGeo& G, const DeviceState& Dref, const ppc::TcLay
   p.tiles_y = G.tiles_y;
   p.ntiles = G.ntiles;
   p.split = G.split;
-  const bool wide = f16 && G.ncols > ACC2;  // single-buffered f16 tile (one per CTA)
+  const bool wide = f16 && G.ncols > ACC2;  // single-buffered f16 tile
   p.nbuf = wide ? 1 : 2;
   p.acc2 = wide ? NMAX : ACC2;
   const int mrows = G.pair ? 2 * FB : FB;  // pairs: one M = 256 MMA over both CTAs' filter blocks
